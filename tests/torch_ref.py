@@ -1,0 +1,66 @@
+"""Independent fp64 CPU model built from torch.nn library layers (test helper only).
+
+It composes F.layer_norm, F.linear, F.scaled_dot_product_attention, F.gelu and
+F.cross_entropy according to the block equations (Eq. 1, Eq. 2, the FAL+
+equation of App. D.1) and differentiates with autograd.  It shares no code with
+the oracle and none with the CUDA library; tests use it to pin the oracle's
+forward composition and its manual backward.
+"""
+from __future__ import annotations
+
+import torch
+import torch.nn.functional as Fn
+
+
+def _ln(x, p, name):
+    d = x.shape[-1]
+    return Fn.layer_norm(x, (d,), p[name + ".g"], p[name + ".b"], eps=1e-5)
+
+
+def _mha(x, p, i, H):
+    B, T, d = x.shape
+    qkv = Fn.linear(x, p[f"h{i}.attn.w_qkv"], p[f"h{i}.attn.b_qkv"])
+    q, k, v = qkv.split(d, dim=-1)
+    sh = lambda t: t.reshape(B, T, H, d // H).transpose(1, 2)
+    o = Fn.scaled_dot_product_attention(sh(q), sh(k), sh(v), is_causal=True)
+    o = o.transpose(1, 2).reshape(B, T, d)
+    return Fn.linear(o, p[f"h{i}.attn.w_o"], p[f"h{i}.attn.b_o"])
+
+
+def _mlp(x, p, i):
+    h = Fn.linear(x, p[f"h{i}.mlp.w_up"], p[f"h{i}.mlp.b_up"])
+    return Fn.linear(Fn.gelu(h, approximate="tanh"), p[f"h{i}.mlp.w_down"], p[f"h{i}.mlp.b_down"])
+
+
+def model_loss(params, variant, heads, tokens, targets, layers, parallel=False):
+    """Mean next-token loss.  ``parallel=True`` builds the GPT-J style block
+    X + MHA(LN1(X)) + MLP(LN1(X)) (no first-attention term)."""
+    p = params
+    tok = torch.as_tensor(tokens, dtype=torch.long)
+    B, T = tok.shape
+    X = Fn.embedding(tok, p["wte"]) + p["wpe"][:T][None]
+    a1 = None
+    for i in range(layers):
+        n1 = _ln(X, p, f"h{i}.ln1")
+        a = _mha(n1, p, i, heads)
+        if i == 0:
+            a1 = a
+        if parallel:
+            m = n1
+        elif variant == "fal":
+            m = n1 + _ln(a1, p, "lnF")
+        else:
+            m = _ln(X + a, p, f"h{i}.ln2")
+            if variant == "falplus" and i >= 1:
+                m = m + _ln(a1, p, f"h{i}.lnF")
+        X = X + a + _mlp(m, p, i)
+    xf = _ln(X, p, "lnf")
+    logits = xf @ p["wte"].T
+    return Fn.cross_entropy(logits.reshape(B * T, -1), torch.as_tensor(targets, dtype=torch.long).reshape(-1))
+
+
+def loss_and_grads(params_np, variant, heads, tokens, targets, layers, parallel=False):
+    p = {k: torch.tensor(v, dtype=torch.float64, requires_grad=True) for k, v in params_np.items()}
+    loss = model_loss(p, variant, heads, tokens, targets, layers, parallel)
+    loss.backward()
+    return float(loss), {k: t.grad.numpy() if t.grad is not None else torch.zeros_like(t).numpy() for k, t in p.items()}
