@@ -1,0 +1,161 @@
+/*
+ * fal.h - C ABI of the GB300 (sm_103a) training hot path for decoder stacks of
+ * GPT (Pre-LN), FAL and FAL+ blocks ("First Attentions Last", arXiv 2510.14614).
+ *
+ * Block equations implemented (paper section / equation):
+ *   GPT  (Eq. 1, Sec. 2):   X_{i+1} = X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i + MHA_i(LN(X_i))))
+ *   FAL  (Eq. 2, Sec. 4.1): X_{i+1} = X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i) + LN_F(MHA_1(LN(X_1))))
+ *        LN(X_i) is the same LayerNorm output that feeds MHA_i; LN_F is one
+ *        LayerNorm shared by all blocks (applied "only once", Sec. 4.1).
+ *   FAL+ (Sec. 5, App. D.1): block 1 is the standard block; block i >= 2 feeds
+ *        MLP_i(LN(X_i + MHA_i(LN(X_i))) + LN_{F,i}(MHA_1(LN(X_1)))).
+ * GPT-2 conventions: learned positions, tied LM head, final LN, biases on every
+ * linear map, tanh GELU, LN eps 1e-5, causal attention scaled by 1/sqrt(head_dim),
+ * mean token cross-entropy; AdamW with bias correction and decoupled weight
+ * decay on matrices and embeddings (App. A: lr 1e-4, weight decay 1e-3).
+ *
+ * Conventions for every entry point:
+ *   - Return 0 (FAL_OK) or a positive FAL_ERR_* code; nothing aborts or throws.
+ *   - A non-OK return leaves a message retrievable with fal_last_error().
+ *   - "device or host" pointers are resolved through unified addressing
+ *     (cudaMemcpyDefault); host memory should be pinned for asynchronous copies.
+ *   - All work is enqueued on the caller's streams; only calls that return a
+ *     host value (a loss, parameters, a tap) or fal_sync() synchronize.
+ */
+#ifndef FAL_H
+#define FAL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* status codes */
+#define FAL_OK 0
+#define FAL_ERR_ARG 1         /* null pointer, bad shape, bad alignment, token id out of range */
+#define FAL_ERR_STATE 2       /* call order (e.g. backward without a forward) */
+#define FAL_ERR_WORKSPACE 3   /* workspace smaller than fal_workspace_size() */
+#define FAL_ERR_CUDA 4        /* a CUDA runtime/driver call failed */
+#define FAL_ERR_TIMEOUT 5     /* a bounded device-side wait expired (kernel returned early) */
+#define FAL_ERR_UNSUPPORTED 6 /* configuration valid but not implemented on this path */
+
+/* block variants */
+#define FAL_GPT 0
+#define FAL_FAL 1
+#define FAL_FALPLUS 2
+
+/* arithmetic of the path */
+#define FAL_BF16 0        /* bf16 tensor-core GEMMs/attention, fp32 accumulation, fp32 residual */
+#define FAL_FP32_DEBUG 1  /* plain fp32 FMA kernels everywhere (no TF32), for parity at 1e-4 */
+
+/* schedule of the two branches of a FAL block (Sec. 4.2 "Single-GPU Acceleration") */
+#define FAL_SCHED_SERIAL 0      /* one stream, MHA branch then MLP branch */
+#define FAL_SCHED_TWO_STREAM 1  /* FAL blocks i >= 2: MHA branch on stream_side, MLP on stream_main */
+
+typedef struct fal_config {
+    int variant;      /* FAL_GPT | FAL_FAL | FAL_FALPLUS */
+    int layers;       /* L >= 1 */
+    int d_model;      /* d, multiple of 8 (bf16) or 4 (fp32 debug) */
+    int heads;        /* H, d % H == 0; bf16 needs head_dim in {64, 128} */
+    int d_ff;         /* MLP width, multiple of 8 */
+    int seq;          /* T >= 1 (positions table size) */
+    int batch;        /* B >= 1 */
+    int vocab;        /* V >= 2 */
+    int precision;    /* FAL_BF16 | FAL_FP32_DEBUG */
+    int schedule;     /* FAL_SCHED_* */
+    float lr, beta1, beta2, eps, weight_decay;  /* AdamW */
+} fal_config;
+
+typedef struct fal_tensor_info {
+    char name[48];   /* e.g. "wte", "h3.attn.w_qkv", "lnF.g" (layers numbered from 0) */
+    size_t offset;   /* first element inside the flat fp32 parameter buffer */
+    size_t numel;
+    int ndim;        /* 1 or 2 */
+    int shape[2];    /* matrices are [out, in], row-major */
+    int decayed;     /* 1 if AdamW applies weight decay */
+} fal_tensor_info;
+
+typedef struct fal_handle fal_handle;
+
+/* Bytes of device workspace a configuration needs (parameters, gradients,
+ * AdamW moments, bf16 weight copy, activations, scratch).  Error: FAL_ERR_ARG. */
+int fal_workspace_size(const fal_config* cfg, size_t* bytes);
+
+/* Creates a model inside `workspace` (device memory owned by the caller, at
+ * least fal_workspace_size() bytes, 256-byte aligned).  stream_main and
+ * stream_side are cudaStream_t values owned by the caller (may be equal; NULL
+ * means the legacy default stream).  Parameters start at zero: load them with
+ * fal_set_params().  The handle owns only host memory, CUDA events and TMA
+ * descriptors; fal_destroy() releases them. */
+int fal_create(const fal_config* cfg, void* workspace, size_t bytes,
+               void* stream_main, void* stream_side, fal_handle** out);
+void fal_destroy(fal_handle* h);
+
+/* Forward pass and mean cross-entropy loss over B*T positions.
+ * tokens, targets: int32 [B, T] row-major, device or host.  loss_host may be
+ * NULL (the loss stays on the device, see fal_get_loss); otherwise the call
+ * synchronizes and writes it.  Token ids outside [0, V) are zeroed and
+ * reported as FAL_ERR_ARG at the next synchronizing call. */
+int fal_forward(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host);
+
+/* Gradients of the last forward's loss into the flat fp32 gradient buffer
+ * (overwritten, not accumulated).  FAL_ERR_STATE without a preceding forward. */
+int fal_backward(fal_handle* h);
+
+/* One AdamW step over the flat parameter buffer; also refreshes the bf16
+ * weight copy.  FAL_ERR_STATE without a preceding backward. */
+int fal_step(fal_handle* h);
+
+/* forward + backward + step. */
+int fal_train_step(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host);
+
+/* Waits for both streams and reports device-side errors (token range, wait timeouts). */
+int fal_sync(fal_handle* h);
+
+/* Loss of the last forward (synchronizes). */
+int fal_get_loss(fal_handle* h, float* loss_host);
+
+/* Parameter table: n_tensors entries describing the flat buffer of n_elems floats. */
+int fal_param_count(fal_handle* h, int* n_tensors, size_t* n_elems);
+int fal_param_info(fal_handle* h, int idx, fal_tensor_info* info);
+
+/* Copy the whole flat fp32 buffer (n must equal n_elems); src/dst device or host.
+ * fal_set_params also refreshes the bf16 weight copy and resets AdamW state. */
+int fal_set_params(fal_handle* h, const float* src, size_t n);
+int fal_get_params(fal_handle* h, float* dst, size_t n);
+int fal_get_grads(fal_handle* h, float* dst, size_t n);
+
+/* Debug view of a saved activation of the last forward, converted to fp32.
+ * name in {"X","u","m","qkv","ctx","h","g","Y","a1","xf","logits"}; layer is
+ * ignored for the global ones ("a1","xf","logits"; "X" with layer==L is the
+ * stack output).  n must equal the tensor's element count (logits: B*T*V). */
+int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n);
+
+/* Live kernel timing for roofline reports.  While enabled, every GEMM and
+ * attention launch of this handle is bracketed by CUDA events on its own
+ * stream (no synchronization is added).  fal_profile_read() synchronizes,
+ * sums the event intervals since the last read, and resets the counters.
+ * FLOPs are algorithmic: 2*M*N*K per GEMM; causal attention counts half of
+ * the dense 4*B*H*T^2*hd forward and twice that for the backward. */
+typedef struct fal_profile {
+    double gemm_ms, gemm_flops;
+    long long gemm_launches;
+    double attn_ms, attn_flops;
+    long long attn_launches;
+} fal_profile;
+int fal_profile_enable(fal_handle* h, int enable);
+int fal_profile_read(fal_handle* h, fal_profile* out);
+
+/* Number of kernels this library has launched in this process (all handles). */
+long long fal_launch_count(void);
+
+/* Message for the last failed call on this handle (never NULL). */
+const char* fal_last_error(const fal_handle* h);
+const char* fal_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FAL_H */

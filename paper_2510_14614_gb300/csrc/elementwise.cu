@@ -1,0 +1,458 @@
+// Bandwidth-bound kernels of the path: embedding gather/scatter, LayerNorm
+// forward/backward (one warp per row, 128-bit vector access, warp-shuffle
+// reductions), column reductions for LN/bias gradients, the cross-entropy
+// head, and AdamW over the flat parameter buffer.
+#include "common.cuh"
+#include "internal.h"
+
+namespace fal {
+
+namespace {
+
+constexpr float LN_EPS = 1e-5f;
+
+// ------------------------------------------------------------ embedding
+__global__ void embed_fwd_kernel(int rows, int T, int d, int V, const int32_t* __restrict__ tok,
+                                 const float* __restrict__ wte, const float* __restrict__ wpe, float* __restrict__ X,
+                                 int* err) {
+  const int r = blockIdx.x;
+  if (r >= rows) return;
+  int id = tok[r];
+  const bool bad = id < 0 || id >= V;
+  if (bad) {
+    if (threadIdx.x == 0) set_dev_err(err, DEV_ERR_TOKEN);
+  }
+  const int t = r % T;
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
+    float4 e = bad ? make_float4(0.f, 0.f, 0.f, 0.f) : load4(wte + (long)id * d + c);
+    float4 p = load4(wpe + (long)t * d + c);
+    store4(X + (long)r * d + c, make_float4(e.x + p.x, e.y + p.y, e.z + p.z, e.w + p.w));
+  }
+}
+
+__global__ void embed_bwd_tok_kernel(int rows, int d, const int32_t* __restrict__ tok, const float* __restrict__ dX,
+                                     float* __restrict__ dwte, int V) {
+  const int r = blockIdx.x;
+  const int id = tok[r];
+  if (id < 0 || id >= V) return;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) atomicAdd(dwte + (long)id * d + c, dX[(long)r * d + c]);
+}
+
+__global__ void embed_bwd_pos_kernel(int B, int T, int d, const float* __restrict__ dX, float* __restrict__ dwpe) {
+  const long n = (long)T * d;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    float s = 0.f;
+    for (int b = 0; b < B; ++b) s += dX[(long)b * n + i];
+    dwpe[i] = s;
+  }
+}
+
+// ------------------------------------------------------------ LayerNorm
+// NV float4 per lane covers up to NV*128 columns.
+template <typename act_t, int NV>
+__global__ void __launch_bounds__(256) ln_fwd_kernel(LnFwdArgs a) {
+  const int warps = blockDim.x / 32;
+  const int row = blockIdx.x * warps + threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (row >= a.rows) return;
+  const int d = a.d;
+  const float* x = a.x + (long)row * d;
+  float4 v[NV];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    v[i] = (c < d) ? load4(x + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    s += v[i].x + v[i].y + v[i].z + v[i].w;
+  }
+  const float mean = warp_sum(s) / d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    if (c < d) {
+      const float dx = v[i].x - mean, dy = v[i].y - mean, dz = v[i].z - mean, dw = v[i].w - mean;
+      q += dx * dx + dy * dy + dz * dz + dw * dw;
+    }
+  }
+  const float rstd = rsqrtf(warp_sum(q) / d + LN_EPS);
+  if (lane == 0) {
+    if (a.mean) a.mean[row] = mean;
+    if (a.rstd) a.rstd[row] = rstd;
+  }
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    if (c >= d) continue;
+    float4 y = make_float4((v[i].x - mean) * rstd, (v[i].y - mean) * rstd, (v[i].z - mean) * rstd, (v[i].w - mean) * rstd);
+    if (a.gamma) {
+      const float4 g = load4(a.gamma + c), b = load4(a.beta + c);
+      y = make_float4(y.x * g.x + b.x, y.y * g.y + b.y, y.z * g.z + b.z, y.w * g.w + b.w);
+    }
+    if (a.out) store4(reinterpret_cast<act_t*>(a.out) + (long)row * d + c, y);
+    if (a.out_f32) store4(a.out_f32 + (long)row * d + c, y);
+    if (a.out2) {
+      float4 z = load4(a.add_src + (long)row * d + c);
+      if (a.add_g) { const float4 g = load4(a.add_g + c); z = make_float4(z.x * g.x, z.y * g.y, z.z * g.z, z.w * g.w); }
+      if (a.add_b) { const float4 b = load4(a.add_b + c); z = make_float4(z.x + b.x, z.y + b.y, z.z + b.z, z.w + b.w); }
+      store4(reinterpret_cast<act_t*>(a.out2) + (long)row * d + c, make_float4(y.x + z.x, y.y + z.y, y.z + z.z, y.w + z.w));
+    }
+  }
+}
+
+// dx = rstd * (gdy - mean(gdy) - xhat * mean(gdy * xhat)) + dres, gdy = (dy + dy2) * gamma
+template <typename act_t, int NV>
+__global__ void __launch_bounds__(256) ln_bwd_kernel(LnBwdArgs a) {
+  const int warps = blockDim.x / 32;
+  const int row = blockIdx.x * warps + threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (row >= a.rows) return;
+  const int d = a.d;
+  const long off = (long)row * d;
+  const float mean = a.mean[row], rstd = a.rstd[row];
+  float4 xh[NV], gd[NV];
+  float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    if (c < d) {
+      float4 x = load4(a.x + off + c);
+      xh[i] = make_float4((x.x - mean) * rstd, (x.y - mean) * rstd, (x.z - mean) * rstd, (x.w - mean) * rstd);
+      float4 g = load4(a.dy + off + c);
+      if (a.dy2) { float4 g2 = load4(a.dy2 + off + c); g = make_float4(g.x + g2.x, g.y + g2.y, g.z + g2.z, g.w + g2.w); }
+      if (a.gamma) { float4 w = load4(a.gamma + c); g = make_float4(g.x * w.x, g.y * w.y, g.z * w.z, g.w * w.w); }
+      gd[i] = g;
+      s1 += g.x + g.y + g.z + g.w;
+      s2 += g.x * xh[i].x + g.y * xh[i].y + g.z * xh[i].z + g.w * xh[i].w;
+    } else {
+      xh[i] = gd[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 4;
+    if (c >= d) continue;
+    float4 r = make_float4(rstd * (gd[i].x - m1 - xh[i].x * m2), rstd * (gd[i].y - m1 - xh[i].y * m2),
+                           rstd * (gd[i].z - m1 - xh[i].z * m2), rstd * (gd[i].w - m1 - xh[i].w * m2));
+    if (a.dres) { float4 q = load4(a.dres + off + c); r = make_float4(r.x + q.x, r.y + q.y, r.z + q.z, r.w + q.w); }
+    store4(a.dx + off + c, r);
+    if (a.dx_act) store4(reinterpret_cast<act_t*>(a.dx_act) + off + c, r);
+  }
+}
+
+// ------------------------------------------------------------ column sums
+constexpr int CS_COLS = 256;   // columns per block (one per thread)
+constexpr int CS_CHUNKS = 64;  // row chunks (partials)
+
+template <typename act_t>
+__global__ void __launch_bounds__(CS_COLS) colsum_kernel(ColsumArgs a) {
+  const int c = blockIdx.x * CS_COLS + threadIdx.x;
+  const int chunk = blockIdx.y;
+  const int per = (a.rows + CS_CHUNKS - 1) / CS_CHUNKS;
+  const int r0 = chunk * per, r1 = min(a.rows, r0 + per);
+  if (c >= a.d) return;
+  float s0 = 0.f, s1 = 0.f;
+  for (int r = r0; r < r1; ++r) {
+    float v = a.src_act ? to_f(reinterpret_cast<const act_t*>(a.src)[(long)r * a.ld + c])
+                        : reinterpret_cast<const float*>(a.src)[(long)r * a.ld + c];
+    if (a.src2) v += a.src2[(long)r * a.ld + c];
+    s0 += v;
+    if (a.bmode == 1) s1 += v * (a.x[(long)r * a.d + c] - a.mean[r]) * a.rstd[r];
+    else if (a.bmode == 2) s1 += v * a.bsrc[(long)r * a.d + c];
+  }
+  a.partial[((long)chunk * 2 + 0) * a.d + c] = s0;
+  a.partial[((long)chunk * 2 + 1) * a.d + c] = s1;
+}
+
+__global__ void colsum_finish_kernel(ColsumArgs a) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= a.d) return;
+  float s0 = 0.f, s1 = 0.f;
+  for (int k = 0; k < CS_CHUNKS; ++k) {
+    s0 += a.partial[((long)k * 2 + 0) * a.d + c];
+    s1 += a.partial[((long)k * 2 + 1) * a.d + c];
+  }
+  if (a.accumulate) {
+    if (a.out0) a.out0[c] += s0;
+    if (a.out0b) a.out0b[c] += s0;
+    if (a.out1) a.out1[c] += s1;
+  } else {
+    if (a.out0) a.out0[c] = s0;
+    if (a.out0b) a.out0b[c] = s0;
+    if (a.out1) a.out1[c] = s1;
+  }
+}
+
+// ------------------------------------------------------------ cross-entropy
+// One CTA per row: pass 1 online max/sum-exp, pass 2 dlogits = (softmax - onehot)/rows.
+template <typename act_t>
+__global__ void __launch_bounds__(256) ce_kernel(int rows, int V, long ld, const act_t* __restrict__ logits,
+                                                 const int32_t* __restrict__ tgt, act_t* __restrict__ dlogits,
+                                                 float* __restrict__ loss_rows, int* err) {
+  const int r = blockIdx.x;
+  const act_t* x = logits + (long)r * ld;
+  act_t* dx = dlogits + (long)r * ld;
+  float m = -INFINITY, s = 0.f;
+  const int V4 = V & ~3;
+  for (int c = threadIdx.x * 4; c < V4; c += blockDim.x * 4) {
+    const float4 v = load4(x + c);
+    const float mx = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+    if (mx > m) { s *= __expf(m - mx); m = mx; }
+    s += __expf(v.x - m) + __expf(v.y - m) + __expf(v.z - m) + __expf(v.w - m);
+  }
+  for (int c = V4 + threadIdx.x; c < V; c += blockDim.x) {
+    const float v = to_f(x[c]);
+    if (v > m) { s *= __expf(m - v); m = v; }
+    s += __expf(v - m);
+  }
+  __shared__ float sm[32], ss[32];
+  // warp combine
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    const float mn = fmaxf(m, m2);
+    s = (m == -INFINITY ? 0.f : s * __expf(m - mn)) + (m2 == -INFINITY ? 0.f : s2 * __expf(m2 - mn));
+    m = mn;
+  }
+  const int w = threadIdx.x / 32, lane = threadIdx.x % 32, nw = blockDim.x / 32;
+  if (lane == 0) { sm[w] = m; ss[w] = s; }
+  __syncthreads();
+  if (w == 0) {
+    m = lane < nw ? sm[lane] : -INFINITY;
+    s = lane < nw ? ss[lane] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+      const float mn = fmaxf(m, m2);
+      s = (m == -INFINITY ? 0.f : s * __expf(m - mn)) + (m2 == -INFINITY ? 0.f : s2 * __expf(m2 - mn));
+      m = mn;
+    }
+    if (lane == 0) { sm[0] = m; ss[0] = s; }
+  }
+  __syncthreads();
+  m = sm[0];
+  const float inv = 1.f / ss[0];
+  int t = tgt[r];
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0) set_dev_err(err, DEV_ERR_TOKEN);
+    t = -1;
+  }
+  if (threadIdx.x == 0) loss_rows[r] = (m + logf(ss[0])) - (t >= 0 ? to_f(x[t]) : 0.f);
+  const float scale = 1.f / rows;
+  for (int c = threadIdx.x * 4; c < V4; c += blockDim.x * 4) {
+    const float4 v = load4(x + c);
+    float4 p = make_float4(__expf(v.x - m) * inv, __expf(v.y - m) * inv, __expf(v.z - m) * inv, __expf(v.w - m) * inv);
+    if (t >= c && t < c + 4) {
+      if (t == c) p.x -= 1.f; else if (t == c + 1) p.y -= 1.f; else if (t == c + 2) p.z -= 1.f; else p.w -= 1.f;
+    }
+    store4(dx + c, make_float4(p.x * scale, p.y * scale, p.z * scale, p.w * scale));
+  }
+  for (int c = V4 + threadIdx.x; c < V; c += blockDim.x) {
+    float p = __expf(to_f(x[c]) - m) * inv;
+    if (c == t) p -= 1.f;
+    dx[c] = from_f<act_t>(p * scale);
+  }
+  for (int c = V + threadIdx.x; c < ld; c += blockDim.x) dx[c] = from_f<act_t>(0.f);
+}
+
+__global__ void mean_kernel(int n, const float* __restrict__ x, float* __restrict__ out) {
+  __shared__ float sh[32];
+  float s = 0.f;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) s += x[i];
+  s = warp_sum(s);
+  if (threadIdx.x % 32 == 0) sh[threadIdx.x / 32] = s;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    s = threadIdx.x < blockDim.x / 32 ? sh[threadIdx.x] : 0.f;
+    s = warp_sum(s);
+    if (threadIdx.x == 0) *out = s / n;
+  }
+}
+
+// ------------------------------------------------------------ misc
+__global__ void add_scaled_cols_kernel(long n, int d, const float* __restrict__ src, const float* __restrict__ colvec,
+                                       float* __restrict__ dst) {
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n / 4; i += (long)gridDim.x * blockDim.x) {
+    const long e = i * 4;
+    const int c = e % d;
+    const float4 s = load4(src + e), g = load4(colvec + c);
+    float4 o = load4(dst + e);
+    o.x += s.x * g.x; o.y += s.y * g.y; o.z += s.z * g.z; o.w += s.w * g.w;
+    store4(dst + e, o);
+  }
+}
+
+// p <- p - lr * (mhat / (sqrt(vhat) + eps) + wd * p) for i < n_decay, no decay after;
+// shadow (bf16 copy of p) refreshed in the same pass.
+__global__ void adamw_kernel(size_t n, size_t n_decay, float* __restrict__ p, const float* __restrict__ g,
+                             float* __restrict__ m, float* __restrict__ v, bf16* __restrict__ shadow, float lr,
+                             float b1, float b2, float eps, float wd, float rbc1, float rbc2) {
+  const size_t n4 = n / 4;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
+    const size_t e = i * 4;
+    float4 pp = load4(p + e), gg = load4(g + e), mm = load4(m + e), vv = load4(v + e);
+    float* pa = &pp.x; float* ga = &gg.x; float* ma = &mm.x; float* va = &vv.x;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      ma[j] = b1 * ma[j] + (1.f - b1) * ga[j];
+      va[j] = b2 * va[j] + (1.f - b2) * ga[j] * ga[j];
+      const float mh = ma[j] * rbc1, vh = va[j] * rbc2;
+      const float w = (e + j < n_decay) ? wd : 0.f;
+      pa[j] -= lr * (mh / (sqrtf(vh) + eps) + w * pa[j]);
+    }
+    store4(p + e, pp); store4(m + e, mm); store4(v + e, vv);
+    if (shadow) store4(shadow + e, pp);
+  }
+}
+
+__global__ void f32_to_bf16_kernel(size_t n, const float* __restrict__ s, bf16* __restrict__ d) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+    d[i] = __float2bfloat16_rn(s[i]);
+}
+
+template <typename act_t>
+__global__ void act_to_f32_2d_kernel(int rows, int cols, long ld, const act_t* __restrict__ s, float* __restrict__ d) {
+  const long n = (long)rows * cols;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    const long r = i / cols, c = i % cols;
+    d[i] = to_f(s[r * ld + c]);
+  }
+}
+
+int grid_for(long n, int block) {
+  long g = (n + block - 1) / block;
+  if (g > 8192) g = 8192;
+  if (g < 1) g = 1;
+  return (int)g;
+}
+
+template <typename act_t>
+int ln_fwd_t(const LnFwdArgs& a, cudaStream_t s) {
+  const int nv = (a.d + 127) / 128;
+  const int blocks = (a.rows + 7) / 8;
+  if (nv <= 1) ln_fwd_kernel<act_t, 1><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 2) ln_fwd_kernel<act_t, 2><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 4) ln_fwd_kernel<act_t, 4><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 8) ln_fwd_kernel<act_t, 8><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 16) ln_fwd_kernel<act_t, 16><<<blocks, 256, 0, s>>>(a);
+  else return 6;
+  return 0;
+}
+template <typename act_t>
+int ln_bwd_t(const LnBwdArgs& a, cudaStream_t s) {
+  const int nv = (a.d + 127) / 128;
+  const int blocks = (a.rows + 7) / 8;
+  if (nv <= 1) ln_bwd_kernel<act_t, 1><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 2) ln_bwd_kernel<act_t, 2><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 4) ln_bwd_kernel<act_t, 4><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 8) ln_bwd_kernel<act_t, 8><<<blocks, 256, 0, s>>>(a);
+  else if (nv <= 16) ln_bwd_kernel<act_t, 16><<<blocks, 256, 0, s>>>(a);
+  else return 6;
+  return 0;
+}
+
+int last_err() { return cudaGetLastError() == cudaSuccess ? 0 : 4; }
+
+}  // namespace
+
+int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s) {
+  if (a.rows <= 0) return 0;
+  if (a.d % 4) return 1;
+  int r = act_bf16 ? ln_fwd_t<bf16>(a, s) : ln_fwd_t<float>(a, s);
+  count_launches(1);
+  return r ? r : last_err();
+}
+
+int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
+  if (a.rows <= 0) return 0;
+  if (a.d % 4) return 1;
+  int r = act_bf16 ? ln_bwd_t<bf16>(a, s) : ln_bwd_t<float>(a, s);
+  count_launches(1);
+  return r ? r : last_err();
+}
+
+size_t colsum_partial_floats(int d) { return (size_t)CS_CHUNKS * 2 * d; }
+
+int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
+  if (a.d <= 0) return 0;
+  dim3 grid((a.d + CS_COLS - 1) / CS_COLS, CS_CHUNKS);
+  if (act_bf16) colsum_kernel<bf16><<<grid, CS_COLS, 0, s>>>(a);
+  else colsum_kernel<float><<<grid, CS_COLS, 0, s>>>(a);
+  colsum_finish_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a);
+  count_launches(2);
+  return last_err();
+}
+
+int embed_fwd(int rows, int T, int d, int V, const int32_t* tok, const float* wte, const float* wpe, float* X, int* err,
+              cudaStream_t s) {
+  if (rows <= 0) return 0;
+  if (d % 4) return 1;
+  embed_fwd_kernel<<<rows, 128, 0, s>>>(rows, T, d, V, tok, wte, wpe, X, err);
+  count_launches(1);
+  return last_err();
+}
+
+int embed_bwd(int B, int T, int d, int V, const int32_t* tok, const float* dX, float* dwte, float* dwpe,
+              cudaStream_t s) {
+  const int rows = B * T;
+  if (rows <= 0) return 0;
+  embed_bwd_pos_kernel<<<grid_for((long)T * d, 256), 256, 0, s>>>(B, T, d, dX, dwpe);
+  embed_bwd_tok_kernel<<<rows, 256, 0, s>>>(rows, d, tok, dX, dwte, V);
+  count_launches(2);
+  return last_err();
+}
+
+int cross_entropy(int act_bf16, int rows, int V, long ld, const void* logits, const int32_t* tgt, void* dlogits,
+                  float* loss_rows, float* loss, int* err, cudaStream_t s) {
+  if (rows <= 0) return 0;
+  if (act_bf16)
+    ce_kernel<bf16><<<rows, 256, 0, s>>>(rows, V, ld, reinterpret_cast<const bf16*>(logits), tgt,
+                                         reinterpret_cast<bf16*>(dlogits), loss_rows, err);
+  else
+    ce_kernel<float><<<rows, 256, 0, s>>>(rows, V, ld, reinterpret_cast<const float*>(logits), tgt,
+                                          reinterpret_cast<float*>(dlogits), loss_rows, err);
+  mean_kernel<<<1, 1024, 0, s>>>(rows, loss_rows, loss);
+  count_launches(2);
+  return last_err();
+}
+
+int add_scaled_cols(int rows, int d, const float* src, const float* colvec, float* dst, cudaStream_t s) {
+  const long n = (long)rows * d;
+  if (n <= 0) return 0;
+  if (d % 4) return 1;
+  add_scaled_cols_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(n, d, src, colvec, dst);
+  count_launches(1);
+  return last_err();
+}
+
+int adamw(size_t n, size_t n_decay, float* p, const float* g, float* m, float* v, void* shadow, float lr, float beta1,
+          float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s) {
+  if (n == 0) return 0;
+  if (n % 4) return 1;
+  const int blocks = num_sms() * 8;
+  adamw_kernel<<<blocks, 256, 0, s>>>(n, n_decay, p, g, m, v, reinterpret_cast<bf16*>(shadow), lr, beta1, beta2, eps, wd,
+                                      1.f / bc1, 1.f / bc2);
+  count_launches(1);
+  return last_err();
+}
+
+int f32_to_bf16(size_t n, const float* src, void* dst, cudaStream_t s) {
+  if (n == 0) return 0;
+  f32_to_bf16_kernel<<<grid_for((long)n, 256), 256, 0, s>>>(n, src, reinterpret_cast<bf16*>(dst));
+  count_launches(1);
+  return last_err();
+}
+
+int act_to_f32_2d(int act_bf16, int rows, int cols, long ld, const void* src, float* dst, cudaStream_t s) {
+  const long n = (long)rows * cols;
+  if (n <= 0) return 0;
+  if (act_bf16) act_to_f32_2d_kernel<bf16><<<grid_for(n, 256), 256, 0, s>>>(rows, cols, ld, reinterpret_cast<const bf16*>(src), dst);
+  else act_to_f32_2d_kernel<float><<<grid_for(n, 256), 256, 0, s>>>(rows, cols, ld, reinterpret_cast<const float*>(src), dst);
+  count_launches(1);
+  return last_err();
+}
+
+int act_to_f32(int act_bf16, size_t n, const void* src, float* dst, cudaStream_t s) {
+  return act_to_f32_2d(act_bf16, 1, (int)n, (long)n, src, dst, s);
+}
+
+}  // namespace fal

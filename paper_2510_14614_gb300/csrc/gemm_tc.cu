@@ -1,0 +1,450 @@
+// tcgen05 / TMEM GEMM fed by TMA, for every bf16 contraction of the path
+// (QKV projection, MLP up-projection + GELU, the fused [ctx | g] x [W_o ; W_down]
+// residual GEMM, LM head, and all data/weight-gradient GEMMs of the backward).
+//
+// Design (sm_103a, one CTA per SM, persistent over output tiles):
+//   warp 0      TMA producer: 128x64 A tile + 256x64 B tile per stage (4 stages),
+//               128-byte swizzle, K-major or MN-major operands.
+//   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
+//               issues tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16),
+//               committing each stage back to the producer.
+//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns per chunk, bias /
+//               GELU / dGELU / residual in fp32, stores to global memory; the
+//               second accumulator lets tile t+1's main loop overlap tile t's
+//               epilogue.
+// Every mbarrier wait is bounded (about one second): on expiry the CTA records
+// DEV_ERR_TIMEOUT in the device error word, drains its in-flight copies and
+// MMAs, frees TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cstring>
+#include <mutex>
+
+#include "gemm_epi.cuh"
+
+namespace fal {
+
+namespace {
+
+constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
+constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;   // 16 KB
+constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KB
+constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr int TC_MN_CHUNK_BYTES = 64 * TC_BK * 2;  // one 64-wide MN chunk of an MN-major tile
+constexpr int TC_BAR_BYTES = 256;
+constexpr int TC_SMEM = TC_STAGES * TC_STAGE_BYTES + 1024 + TC_BAR_BYTES;
+constexpr int TC_THREADS = 192;
+constexpr uint64_t TC_WAIT_NS = 1000000000ull;  // bounded waits: 1 s
+
+struct TcGroup {
+  int M, N, m_tiles, n_tiles, tile_start, nseg;
+  int kb[2];
+  int amap[2], bmap[2];
+  int a_mn, b_mn;
+  uint32_t idesc;
+  EpiParams epi;
+};
+
+struct TcParams {
+  CUtensorMap maps[8];
+  TcGroup grp[2];
+  int ngroups, total_tiles;
+  int* err;
+};
+
+// ------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: false if the phase did not complete within TC_WAIT_NS or another
+// role of this CTA already gave up (abort flag in shared memory).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > TC_WAIT_NS) { *abort_flag = 1; return false; }
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+// Shared-memory matrix descriptor (tcgen05 format): start, leading and stride
+// byte offsets (>>4), version 1 at bits 46-48, 128-byte swizzle (2) at bits 61-63.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+#define TMEM_LD32(taddr, r)                                                                          \
+  asm volatile(                                                                                      \
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15," \
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"                     \
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),          \
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),       \
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),    \
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),    \
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])                                            \
+      : "r"(taddr))
+
+__device__ __forceinline__ void decode_tile(const TcParams& p, int tile, int& g, int& m0, int& n0) {
+  g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+  const TcGroup& G = p.grp[g];
+  const int local = tile - G.tile_start;
+  m0 = (local % G.m_tiles) * TC_BM;
+  n0 = (local / G.m_tiles) * TC_BN;
+}
+
+template <typename act_t>
+__global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t bar_base = base + TC_STAGES * TC_STAGE_BYTES;
+  uint8_t* bar_ptr = smem_raw + (bar_base - raw);
+  auto full_bar = [&](int s) { return bar_base + 8u * s; };
+  auto empty_bar = [&](int s) { return bar_base + 8u * (TC_STAGES + s); };
+  auto tfull_bar = [&](int b) { return bar_base + 8u * (2 * TC_STAGES + b); };
+  auto tempty_bar = [&](int b) { return bar_base + 8u * (2 * TC_STAGES + 2 + b); };
+  const uint32_t drain_bar = bar_base + 8u * (2 * TC_STAGES + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_ptr + 8 * (2 * TC_STAGES + 5));
+  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(bar_ptr + 8 * (2 * TC_STAGES + 5) + 4);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+    for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)), "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_mask = 0, issued_par = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < p.total_tiles && ok; tile += gridDim.x) {
+      int g, m0, n0;
+      decode_tile(p, tile, g, m0, n0);
+      const TcGroup& G = p.grp[g];
+      for (int s = 0; s < G.nseg && ok; ++s) {
+        const CUtensorMap* am = &p.maps[G.amap[s]];
+        const CUtensorMap* bm = &p.maps[G.bmap[s]];
+        for (int kb = 0; kb < G.kb[s]; ++kb) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (lane == 0) {
+            const uint32_t fb = full_bar(stage);
+            const uint32_t sa = base + stage * TC_STAGE_BYTES;
+            const uint32_t sb = sa + TC_A_BYTES;
+            const int k0 = kb * TC_BK;
+            mbar_arrive_expect_tx(fb, TC_STAGE_BYTES);
+            if (G.a_mn) {
+              tma_load_2d(sa, am, m0, k0, fb);
+              tma_load_2d(sa + TC_MN_CHUNK_BYTES, am, m0 + 64, k0, fb);
+            } else {
+              tma_load_2d(sa, am, k0, m0, fb);
+            }
+            if (G.b_mn) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) tma_load_2d(sb + j * TC_MN_CHUNK_BYTES, bm, n0 + 64 * j, k0, fb);
+            } else {
+              tma_load_2d(sb, bm, k0, n0, fb);
+            }
+          }
+          __syncwarp();
+          issued_mask |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == TC_STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+    if (!ok) {
+      // Let every copy this CTA issued land before shared memory is released.
+      for (int s = 0; s < TC_STAGES; ++s) {
+        if (!(issued_mask & (1u << s))) continue;
+        const uint32_t par = (issued_par >> s) & 1u;
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(full_bar(s), par) && global_timer_ns() - t0 < TC_WAIT_NS) {}
+      }
+      if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true, issued_any = false;
+    for (int tile = blockIdx.x; tile < p.total_tiles && ok; tile += gridDim.x) {
+      int g, m0, n0;
+      decode_tile(p, tile, g, m0, n0);
+      const TcGroup& G = p.grp[g];
+      if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + acc * TC_BN;
+      uint32_t accum = 0;
+      for (int s = 0; s < G.nseg && ok; ++s) {
+        for (int kb = 0; kb < G.kb[s]; ++kb) {
+          if (!mbar_wait(full_bar(stage), phase, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t sa = base + stage * TC_STAGE_BYTES;
+            const uint32_t sb = sa + TC_A_BYTES;
+#pragma unroll
+            for (int k = 0; k < TC_BK / 16; ++k) {
+              const uint64_t ad = G.a_mn ? smem_desc(sa + k * 2048, TC_MN_CHUNK_BYTES, 1024)
+                                         : smem_desc(sa + k * 32, 16, 1024);
+              const uint64_t bd = G.b_mn ? smem_desc(sb + k * 2048, TC_MN_CHUNK_BYTES, 1024)
+                                         : smem_desc(sb + k * 32, 16, 1024);
+              tc_mma(d_tmem, ad, bd, G.idesc, accum);
+              accum = 1;
+            }
+            tc_commit(empty_bar(stage));
+          }
+          __syncwarp();
+          issued_any = true;
+          if (++stage == TC_STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) break;
+      if (lane == 0) tc_commit(tfull_bar(acc));
+      __syncwarp();
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+    if (!ok && issued_any) {
+      // Wait for this thread's MMAs to finish before TMEM is freed.
+      if (lane == 0) tc_commit(drain_bar);
+      __syncwarp();
+      const uint64_t t0 = global_timer_ns();
+      while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < TC_WAIT_NS) {}
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 2..5)
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < p.total_tiles; tile += gridDim.x) {
+      int g, m0, n0;
+      decode_tile(p, tile, g, m0, n0);
+      const TcGroup& G = p.grp[g];
+      if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag)) break;
+      tc_fence_after();
+      const int row = m0 + q * 32 + lane;
+      for (int c = 0; c < TC_BN / 32; ++c) {
+        const int col0 = n0 + c * 32;
+        if (col0 >= G.N) break;
+        uint32_t r[32];
+        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + c * 32);
+        TMEM_LD32(taddr, r);
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        epi_row<act_t, 32>(G.epi, G.M, G.N, row, col0, v);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty_bar(acc));
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
+  }
+}
+
+// ------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encoder(std::string* msg) {
+  std::call_once(g_encode_once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (!g_encode && msg) *msg = "cuTensorMapEncodeTiled not available from the driver";
+  return g_encode != nullptr;
+}
+
+// 2-D bf16 map over a row-major matrix with `inner` contiguous elements per row.
+bool encode_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld,
+                uint32_t box_inner, uint32_t box_outer, std::string* msg) {
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15) || ((ld * 2) & 15)) {
+    if (msg) *msg = "tcgen05 GEMM operand needs a 16-byte aligned base and a leading dimension multiple of 8";
+    return false;
+  }
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled failed (code " + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
+// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B,
+// A/B major-ness, N>>3 at bits 17-22, M>>4 at bits 24-28.
+uint32_t make_idesc(int a_mn, int b_mn) {
+  uint32_t d = 0;
+  d |= 1u << 4;             // D format: f32
+  d |= 1u << 7;             // A format: bf16
+  d |= 1u << 10;            // B format: bf16
+  d |= (uint32_t)a_mn << 15;
+  d |= (uint32_t)b_mn << 16;
+  d |= (uint32_t)(TC_BN >> 3) << 17;
+  d |= (uint32_t)(TC_BM >> 4) << 24;
+  return d;
+}
+
+bool check_ld(long ld, const void* p) { return p == nullptr || ((ld & 3) == 0 && (reinterpret_cast<uintptr_t>(p) & 15) == 0); }
+
+}  // namespace
+
+namespace {
+std::atomic<long long> g_launches{0};
+}
+void count_launches(long long n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+long long launches_total() { return g_launches.load(std::memory_order_relaxed); }
+
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg) {
+  if (!get_encoder(msg)) return 4;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+    if (e != cudaSuccess) { if (msg) *msg = std::string("gemm_tc smem attribute: ") + cudaGetErrorString(e); return 4; }
+    attr_set = true;
+  }
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  int nmaps = 0, tiles = 0;
+  p.ngroups = c.ngroups;
+  for (int g = 0; g < c.ngroups; ++g) {
+    const GemmGroupDesc& G = c.g[g];
+    TcGroup& T = p.grp[g];
+    T.M = G.M; T.N = G.N; T.nseg = G.nseg;
+    T.m_tiles = (G.M + TC_BM - 1) / TC_BM;
+    T.n_tiles = (G.N + TC_BN - 1) / TC_BN;
+    T.tile_start = tiles;
+    T.epi = G.epi;
+    const EpiParams& e = G.epi;
+    if (!check_ld(e.ldo, e.out) || !check_ld(e.ldo2, e.out2) || !check_ld(e.ldr, e.resid) ||
+        !check_ld(e.ldr2, e.resid2) || !check_ld(e.ldx, e.aux) || !check_ld(0, e.bias) || !check_ld(0, e.bias2)) {
+      if (msg) *msg = "tcgen05 GEMM epilogue pointers must be 16-byte aligned with leading dimensions multiple of 4";
+      return 1;
+    }
+    if (G.nseg < 1 || G.nseg > 2 || G.M <= 0 || G.N <= 0) { if (msg) *msg = "bad GEMM group"; return 1; }
+    T.a_mn = G.seg[0].A.mn_major;
+    T.b_mn = G.seg[0].B.mn_major;
+    for (int sg = 0; sg < G.nseg; ++sg) {
+      const GemmSeg& S = G.seg[sg];
+      if (S.A.mn_major != T.a_mn || S.B.mn_major != T.b_mn || S.K <= 0) {
+        if (msg) *msg = "GEMM segments of one group must share operand majors";
+        return 1;
+      }
+      T.kb[sg] = (S.K + TC_BK - 1) / TC_BK;
+      // A: logical [M, K]
+      if (S.A.mn_major) {
+        if (!encode_map(&p.maps[nmaps], S.A.ptr, G.M, S.K, S.A.ld, 64, TC_BK, msg)) return 1;
+      } else {
+        if (!encode_map(&p.maps[nmaps], S.A.ptr, S.K, G.M, S.A.ld, TC_BK, TC_BM, msg)) return 1;
+      }
+      T.amap[sg] = nmaps++;
+      if (S.B.mn_major) {
+        if (!encode_map(&p.maps[nmaps], S.B.ptr, G.N, S.K, S.B.ld, 64, TC_BK, msg)) return 1;
+      } else {
+        if (!encode_map(&p.maps[nmaps], S.B.ptr, S.K, G.N, S.B.ld, TC_BK, TC_BN, msg)) return 1;
+      }
+      T.bmap[sg] = nmaps++;
+    }
+    T.idesc = make_idesc(T.a_mn, T.b_mn);
+    tiles += T.m_tiles * T.n_tiles;
+  }
+  p.total_tiles = tiles;
+  p.err = dev_err;
+  if (tiles == 0) return 0;
+  const int grid = tiles < num_sms() ? tiles : num_sms();
+  gemm_tc_kernel<bf16><<<grid, TC_THREADS, TC_SMEM, s>>>(p);
+  count_launches(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) { if (msg) *msg = std::string("gemm_tc launch: ") + cudaGetErrorString(e); return 4; }
+  return 0;
+}
+
+}  // namespace fal

@@ -1,0 +1,116 @@
+// Host-side interface between the translation units of libfal.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string>
+
+namespace fal {
+
+// Device error word codes (written with atomicCAS so the first error sticks).
+enum DevErr { DEV_OK = 0, DEV_ERR_TOKEN = 1, DEV_ERR_TIMEOUT = 2 };
+
+// ---------------------------------------------------------------- GEMM
+// Every GEMM of the path is C[M,N] = sum_k A(m,k) * B(n,k) followed by an
+// epilogue.  A operand element (m,k) lives at A[m*ld + k] (K-major) or
+// A[k*ld + m] (MN-major); B operand element (n,k) at B[n*ld + k] (K-major) or
+// B[k*ld + n] (MN-major).  A group may chain two K segments (two operand pairs
+// summed into one accumulator: the fused [ctx | g] x [W_o ; W_down] residual
+// GEMM), and one launch may run two independent groups.
+enum EpiOp { EPI_NONE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
+enum OutMode { OUT_ACT = 0, OUT_F32 = 1, OUT_F32_ACCUM = 2 };
+
+struct EpiParams {
+  int op;        // EpiOp
+  int out_mode;  // OutMode for `out`
+  void* out;  long ldo;
+  void* out2; long ldo2;     // GELU: gelu(v) (activation type); pre_f32: fp32 copy of acc+bias
+  int pre_f32;               // write out2 = acc + bias before the residual is added
+  const float* bias;  const float* bias2;   // per-column (N) fp32 vectors, may be null
+  const float* resid; long ldr;             // fp32 [M, N] added after pre_f32
+  const float* resid2; long ldr2;
+  const void* aux; long ldx;                // DGELU: pre-activation h (activation type)
+};
+
+struct GemmOperand { const void* ptr; long ld; int mn_major; };
+struct GemmSeg { GemmOperand A, B; int K; };
+struct GemmGroupDesc { int M, N; int nseg; GemmSeg seg[2]; EpiParams epi; };
+struct GemmCall { int ngroups; GemmGroupDesc g[2]; };
+
+// Plain fp32-FMA tiled GEMM (debug precision; also a GPU cross-check).
+// in_bf16: operands are bf16 (else fp32); act_bf16: activation outputs bf16.
+int gemm_simt(const GemmCall& c, int in_bf16, int act_bf16, cudaStream_t s, std::string* msg);
+// tcgen05/TMEM GEMM fed by TMA (bf16 operands, fp32 accumulation, bf16 activations).
+int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg);
+
+// ---------------------------------------------------------------- attention
+// qkv: activation [B*T, 3*H*hd] (q | k | v, head-major inside each third);
+// ctx: activation [B*T, H*hd]; lse: fp32 [B, H, T] in log2 units of the scaled scores.
+int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse,
+             cudaStream_t s, std::string* msg);
+// dq_acc: fp32 [B*T, H*hd] scratch, dvec: fp32 [B, H, T] scratch.
+int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
+             const float* lse, const void* dctx, void* dqkv, float* dq_acc, float* dvec,
+             cudaStream_t s, std::string* msg);
+
+// ---------------------------------------------------------------- elementwise
+struct LnFwdArgs {
+  int rows, d;
+  const float* x;                       // fp32 [rows, d]
+  const float* gamma; const float* beta;  // null => no affine
+  void* out;                            // activation [rows, d] or null
+  float* out_f32;                       // fp32 [rows, d] or null
+  float* mean; float* rstd;             // [rows] or null
+  // out2 = LN(x)*gamma+beta + add_src*add_g + add_b  (activation), if out2 != null
+  void* out2; const float* add_src; const float* add_g; const float* add_b;
+};
+int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s);
+
+struct LnBwdArgs {
+  int rows, d;
+  const float* dy; const float* dy2;    // gradient of the LN output (dy2 may be null)
+  const float* x; const float* mean; const float* rstd; const float* gamma;  // gamma null => 1
+  const float* dres;                    // added to dx (residual branch), may be null
+  float* dx;                            // fp32 out
+  void* dx_act;                         // activation copy (may be null)
+};
+int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s);
+
+// Column sums over rows: s1[c] = sum_r a(r,c)*b(r,c), s0[c] = sum_r a(r,c)
+// with a = src (+ src2), b = LN-normalised x (bmode 1) or bsrc (bmode 2).
+struct ColsumArgs {
+  int rows, d;
+  const void* src; int src_act;   // src_act: src is the activation type (else fp32)
+  long ld;
+  const float* src2;              // fp32, same layout, may be null
+  int bmode; const float* x; const float* mean; const float* rstd; const float* bsrc;
+  float* partial;                 // scratch [nchunk, 2, d]
+  float* out1; float* out0; float* out0b;  // destinations (may be null)
+  int accumulate;                 // add into destinations instead of storing
+};
+int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s);
+size_t colsum_partial_floats(int d);
+
+int embed_fwd(int rows, int T, int d, int V, const int32_t* tok, const float* wte, const float* wpe,
+              float* X, int* err, cudaStream_t s);
+int embed_bwd(int B, int T, int d, int V, const int32_t* tok, const float* dX, float* dwte, float* dwpe,
+              cudaStream_t s);
+// logits/dlogits: activation [rows, ld] with V valid columns; loss_rows fp32 [rows].
+int cross_entropy(int act_bf16, int rows, int V, long ld, const void* logits, const int32_t* tgt,
+                  void* dlogits, float* loss_rows, float* loss, int* err, cudaStream_t s);
+// dst += src * colvec (per column), fp32 [rows, d]
+int add_scaled_cols(int rows, int d, const float* src, const float* colvec, float* dst, cudaStream_t s);
+int adamw(size_t n, size_t n_decay, float* p, const float* g, float* m, float* v, void* shadow_bf16,
+          float lr, float beta1, float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s);
+int f32_to_bf16(size_t n, const float* src, void* dst, cudaStream_t s);
+int act_to_f32(int act_bf16, size_t n, const void* src, float* dst, cudaStream_t s);
+// copy [rows, cols] from a strided activation into dense fp32
+int act_to_f32_2d(int act_bf16, int rows, int cols, long ld, const void* src, float* dst, cudaStream_t s);
+
+int num_sms();
+
+// Process-wide count of kernel launches made by the library.
+void count_launches(long long n);
+long long launches_total();
+
+}  // namespace fal

@@ -1,0 +1,146 @@
+"""Whole-model parity on the GPU through the C ABI against the fp64 oracle.
+
+Same seeded inputs on both sides (paper_2510_14614_gb300.synth).  Tolerances
+are per-tensor relative Frobenius errors: 1e-4 on the fp32 debug path, 1e-2 on
+the bf16 path, for the loss, the saved activations (taps) and every gradient.
+"""
+import numpy as np
+import pytest
+
+from helpers import rel_fro
+from oracle import fal_oracle as O
+from paper_2510_14614_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+VARIANTS = synth.VARIANTS
+
+
+def _model(variant, s, schedule="serial"):
+    from paper_2510_14614_gb300 import fal
+    hp = synth.adamw_hparams()
+    cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
+                          precision=s.precision, schedule=schedule, **hp)
+    return fal.Model(cfg)
+
+
+def _check_parity(variant, s, tol, schedule="serial", seed=0, check_taps=True):
+    params = synth.perturb_params(synth.init_params(variant, s, seed), seed)
+    tok, tgt = synth.make_tokens(s, seed)
+    m = _model(variant, s, schedule)
+    m.set_params(params)
+    loss = m.forward(tok, tgt)
+    cfg = O.Config.from_shape(variant, s)
+    loss_o, cache = O.forward(params, cfg, tok, tgt)
+    grads_o = O.backward(params, cfg, cache)
+    errs = {"loss": abs(loss - loss_o) / abs(loss_o)}
+    if check_taps:
+        for i in range(s.layers):
+            c = cache["layers"][i]
+            for name, ref in (("X", cache["X"][i]), ("u", c["u"]), ("m", c["m"]), ("qkv", c["qkv"]),
+                              ("ctx", c["ctx"]), ("h", c["h"]), ("g", c["g"])):
+                errs[f"{name}{i}"] = rel_fro(m.tap(name, i), ref)
+        errs["Xout"] = rel_fro(m.tap("X", s.layers), cache["X"][s.layers])
+        errs["xf"] = rel_fro(m.tap("xf"), cache["xf"])
+        errs["logits"] = rel_fro(m.tap("logits"), cache["logits"])
+        if variant != "gpt":
+            errs["a1"] = rel_fro(m.tap("a1"), cache["a1"])
+    m.backward()
+    g = m.grads()
+    for k in params:
+        errs["d" + k] = rel_fro(g[k], grads_o[k])
+    bad = {k: v for k, v in errs.items() if not v <= tol}
+    assert not bad, (bad, max(errs.values()))
+    return m, params, g
+
+
+# ---------------------------------------------------------------- fp32 debug
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_tiny_fp32_debug_parity(variant):
+    _check_parity(variant, synth.SHAPES["tiny"], 1e-4)
+
+
+def test_tiny_fp32_fal_two_stream_parity():
+    _check_parity("fal", synth.SHAPES["tiny"].replace(layers=3), 1e-4, schedule="two_stream")
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_adamw_step_matches_oracle(variant):
+    s = synth.SHAPES["tiny"]
+    m, params, g = _check_parity(variant, s, 1e-4, check_taps=False)
+    m.step()
+    after = m.params()
+    hp = synth.adamw_hparams()
+    zeros = {k: np.zeros_like(v, dtype=np.float64) for k, v in params.items()}
+    decayed = {n for n, _, dec in synth.param_specs(variant, s) if dec}
+    ref, _, _ = O.adamw_step(params, g, zeros, zeros, 1, hp["lr"], hp["beta1"], hp["beta2"], hp["eps"],
+                             hp["weight_decay"], decayed)
+    for k in params:
+        np.testing.assert_allclose(after[k], ref[k], rtol=2e-6, atol=2e-7, err_msg=k)
+
+
+def test_param_table_matches_canonical_specs():
+    for variant in VARIANTS:
+        s = synth.SHAPES["tiny"].replace(layers=3)
+        m = _model(variant, s)
+        got = {name: (shape, dec) for name, _, _, shape, dec in m.tensors}
+        want = {name: (tuple(shape), dec) for name, shape, dec in synth.param_specs(variant, s)}
+        assert got == want
+
+
+# ---------------------------------------------------------------- bf16
+SMALL = synth.Shape("small_ragged", 3, 128, 2, 512, 80, 2, 1000, "bf16")        # BT=160, V=1000: ragged tiles
+HD128 = synth.Shape("hd128_ragged", 2, 256, 2, 1024, 130, 1, 777, "bf16")
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("s", [SMALL, HD128], ids=lambda s: s.name)
+def test_bf16_parity_small(variant, s):
+    _check_parity(variant, s, 1e-2)
+
+
+def test_bf16_fal_two_stream_parity():
+    _check_parity("fal", SMALL, 1e-2, schedule="two_stream")
+
+
+@pytest.mark.parametrize("variant,shape", [("fal", "gpt2_small"), ("gpt", "gpt2_small"), ("falplus", "gpt2_medium"),
+                                           ("fal", "gpt_1p3b"), ("fal", "gpt2_xl")])
+def test_bf16_parity_full_width(variant, shape):
+    """Full width (d, H, d_ff, V, T) of each benchmark shape, reduced depth/batch."""
+    s = synth.SHAPES[shape].replace(layers=2, batch=1)
+    _check_parity(variant, s, 1e-2, check_taps=False)
+
+
+def test_token_out_of_range_is_reported():
+    from paper_2510_14614_gb300 import fal
+    s = SMALL
+    m = _model("fal", s)
+    m.set_params(synth.init_params("fal", s, 0))
+    tok, tgt = synth.make_tokens(s, 0)
+    tok[0, 3] = s.vocab + 5
+    with pytest.raises(fal.FalError) as e:
+        m.forward(tok, tgt)
+    assert e.value.code == fal.FAL_ERR_ARG
+    tok[0, 3] = 1
+    assert np.isfinite(m.forward(tok, tgt))  # the handle stays usable
+
+
+def test_call_order_errors():
+    from paper_2510_14614_gb300 import fal
+    m = _model("gpt", SMALL)
+    with pytest.raises(fal.FalError) as e:
+        m.backward()
+    assert e.value.code == fal.FAL_ERR_STATE
+    with pytest.raises(fal.FalError) as e:
+        m.step()
+    assert e.value.code == fal.FAL_ERR_STATE
+
+
+def test_training_reduces_loss():
+    s = SMALL
+    from paper_2510_14614_gb300 import fal
+    m = _model("fal", s)
+    m.set_params(synth.init_params("fal", s, 0))
+    tok, tgt = synth.make_tokens(s, 0)
+    losses = [m.train_step(tok, tgt) for _ in range(6)]
+    assert losses[-1] < losses[0]
