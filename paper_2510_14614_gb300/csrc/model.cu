@@ -68,6 +68,7 @@ struct fal_handle {
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   std::string err;
   int state = 0;  // 0 fresh, 1 after forward, 2 after backward
+  bool has_loss = false;
   long step_t = 0;
 
   std::vector<fal_tensor_info> tensors;
@@ -797,7 +798,7 @@ int fal_sync(fal_handle* h) {
 
 int fal_get_loss(fal_handle* h, float* loss_host) {
   if (!h || !loss_host) return FAL_ERR_ARG;
-  if (h->state < 1) return fail(h, FAL_ERR_STATE, "no forward pass yet");
+  if (!h->has_loss) return fail(h, FAL_ERR_STATE, "no forward pass yet");
   int r = read_dev_err(h);
   if (r) return r;
   if (cudaMemcpy(loss_host, h->loss, sizeof(float), cudaMemcpyDeviceToHost) != cudaSuccess)
@@ -810,6 +811,7 @@ int fal_forward(fal_handle* h, const int32_t* tokens, const int32_t* targets, fl
   int r = forward_impl(h, tokens, targets);
   if (r) return r;
   h->state = 1;
+  h->has_loss = true;
   if (loss_host) {
     if (cudaMemcpyAsync(loss_host, h->loss, sizeof(float), cudaMemcpyDeviceToHost, h->sm) != cudaSuccess)
       return fail(h, FAL_ERR_CUDA, "loss copy failed");

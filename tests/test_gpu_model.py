@@ -144,3 +144,4 @@ def test_training_reduces_loss():
     tok, tgt = synth.make_tokens(s, 0)
     losses = [m.train_step(tok, tgt) for _ in range(6)]
     assert losses[-1] < losses[0]
+    assert m.loss() == losses[-1]  # the last forward's loss stays readable after the step
