@@ -44,6 +44,29 @@ size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd);
 int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
                              const void* dctx, void* dqkv, float* scratch, void* stream);
 
+/* Allocation-free variant of fal_kernel_attention_bwd (the paper has no
+ * counterpart: this is a deployment convenience).  It is for callers that may
+ * not allocate device memory themselves -- for instance code running inside a
+ * host framework that owns every device byte through its own pool and forbids
+ * stray cudaMalloc/cudaFree (which also synchronize the device), or callers
+ * that simply cannot pass a scratch buffer.  Same arguments as
+ * fal_kernel_attention_bwd minus `scratch`; same results.
+ *
+ * Scratch comes from one fixed array of FAL_NOALLOC_ATTN_SCRATCH_FLOATS fp32
+ * values (16 MiB) compiled into libfal.so: every GPU that loads the library
+ * holds it until the process exits.  The call needs
+ * B*T*H*hd + B*H*T <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS and returns
+ * FAL_ERR_WORKSPACE (launching nothing) above that.  It never calls cudaMalloc,
+ * cudaFree or any allocating routine.  The first call on each device looks up
+ * the array's device address (cudaGetSymbolAddress, with that device current);
+ * make that first call before any stream capture.  All calls share the one
+ * array and each call clears what it needs, so calls that overlap on the GPU
+ * (different streams, or several host threads on one device) race: serialize
+ * them. */
+#define FAL_NOALLOC_ATTN_SCRATCH_FLOATS (4u * 1024u * 1024u)
+int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
+                                     const void* dctx, void* dqkv, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -624,3 +624,56 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
 }
 
 }  // namespace fal
+
+// ------------------------------------------------------------ allocation-free entry point
+// Scratch for fal_kernel_attention_bwd_noalloc: a fixed file-scope device array
+// (dQ accumulator followed by the D = rowsum(dO * O) vector).  Host code only
+// ever sees a stand-in for this symbol, so its device address is looked up
+// once per device with cudaGetSymbolAddress while that device is current.
+#include <mutex>
+
+#include "../../include/fal.h"
+#include "../../include/fal_kernels.h"
+
+namespace {
+
+constexpr size_t kNoAllocFloats = FAL_NOALLOC_ATTN_SCRATCH_FLOATS;
+static __device__ __align__(256) float g_noalloc_attn_scratch[kNoAllocFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (looked up once).
+int noalloc_scratch(float** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FAL_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return FAL_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_attn_scratch) != cudaSuccess || !p) return FAL_ERR_CUDA;
+    g_noalloc_ptr[dev] = static_cast<float*>(p);
+  }
+  *out = g_noalloc_ptr[dev];
+  return FAL_OK;
+}
+
+}  // namespace
+
+extern "C" int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, const void* qkv, const void* ctx,
+                                                const float* lse, const void* dctx, void* dqkv, void* stream) {
+  if (B < 0 || T < 0 || H <= 0 || hd <= 0 || !qkv || !ctx || !lse || !dctx || !dqkv) return FAL_ERR_ARG;
+  const size_t dq_floats = (size_t)B * T * H * hd;
+  const size_t need = dq_floats + (size_t)B * H * T;
+  if (need > kNoAllocFloats) return FAL_ERR_WORKSPACE;
+  float* scratch = nullptr;
+  const int rc = noalloc_scratch(&scratch);
+  if (rc != FAL_OK) return rc;
+  std::string msg;
+  // attn_bwd's first kernel zeroes the dQ accumulator and writes every D entry,
+  // so nothing left in the shared array by an earlier call leaks into this one.
+  const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, scratch + dq_floats,
+                              reinterpret_cast<cudaStream_t>(stream), &msg);
+  return r == 0 ? FAL_OK : r == 1 ? FAL_ERR_ARG : r == 6 ? FAL_ERR_UNSUPPORTED : FAL_ERR_CUDA;
+}

@@ -75,6 +75,7 @@ _SIGS = {
     "fal_kernel_attention_fwd": (ctypes.c_int, [ctypes.c_int] * 4 + [ctypes.c_void_p] * 4),
     "fal_kernel_attention_bwd_scratch": (ctypes.c_size_t, [ctypes.c_int] * 4),
     "fal_kernel_attention_bwd": (ctypes.c_int, [ctypes.c_int] * 4 + [ctypes.c_void_p] * 7),
+    "fal_kernel_attention_bwd_noalloc": (ctypes.c_int, [ctypes.c_int] * 4 + [ctypes.c_void_p] * 6),
 }
 
 
