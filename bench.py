@@ -44,7 +44,18 @@ def parse():
     ap.add_argument("--schedule", default="two_stream", choices=["serial", "two_stream"])
     ap.add_argument("--no-baseline", action="store_true", help="skip the same-library GPT baseline")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--layers", type=int, default=None, help="override depth (small profiling cases only)")
+    ap.add_argument("--batch", type=int, default=None, help="override batch (small profiling cases only)")
     return ap.parse_args()
+
+
+def shape_of(args):
+    s = synth.SHAPES[args.workload]
+    if args.layers:
+        s = s.replace(layers=args.layers, name=f"{s.name}_L{args.layers}")
+    if args.batch:
+        s = s.replace(batch=args.batch, name=f"{s.name}_B{args.batch}")
+    return s
 
 
 def dist_env():
@@ -109,7 +120,7 @@ def cpu_cores():
 
 
 def run_reference(args, n):
-    s = synth.SHAPES[args.workload]
+    s = shape_of(args)
     for _ in range(args.warmup):
         oracle_step_sample(s, args.variant)
     times = []
@@ -286,7 +297,7 @@ def main():
     dev = torch.device(f"cuda:{local}")
     fal.lib()
     peaks, peak_kind = measured_peaks()
-    s = synth.SHAPES[args.workload]
+    s = shape_of(args)
     main_res = time_variant(args, s, args.variant, args.schedule, torch, fal, dev, n, world, rank, peaks, True)
     base = None
     if not args.no_baseline and args.variant != "gpt":

@@ -14,8 +14,9 @@
 extern "C" {
 #endif
 
-#define FAL_ENGINE_TCGEN05 0  /* tcgen05/TMEM GEMM fed by TMA (bf16 operands only) */
-#define FAL_ENGINE_SIMT 1     /* plain fp32-FMA tiled GEMM */
+#define FAL_ENGINE_TCGEN05 0       /* tcgen05/TMEM GEMM fed by TMA, one CTA per 128x256 tile (used by the model) */
+#define FAL_ENGINE_SIMT 1         /* plain fp32-FMA tiled GEMM */
+#define FAL_ENGINE_TCGEN05_PAIR 2  /* tcgen05/TMEM GEMM fed by TMA, CTA pairs (cta_group::2, 256x256 tiles) */
 
 /* C[M,N] = sum_k A(m,k) B(n,k) (+ bias[n]) : the contraction of every linear map
  * of the blocks (Eq. 1, Eq. 2) and of their gradients.
@@ -23,7 +24,7 @@ extern "C" {
  *   B(n,k) = B[n*ldb + k] if !b_mn_major else B[k*ldb + n]
  * A, B: bf16 (in_f32 = 0) or fp32 (in_f32 = 1; SIMT engine only).
  * C: bf16 (c_f32 = 0) or fp32 (c_f32 = 1), row-major with leading dim ldc.
- * bias: fp32 [N] or NULL.  tcgen05 engine: A, B, C, bias 16-byte aligned,
+ * bias: fp32 [N] or NULL.  tcgen05 engines: A, B, C, bias 16-byte aligned,
  * lda/ldb multiples of 8, ldc a multiple of 4.  dev_err: device int that
  * receives a nonzero code if a bounded wait inside the kernel expires (may be NULL).
  * Errors: FAL_ERR_ARG (shape/alignment), FAL_ERR_CUDA (launch). */

@@ -53,6 +53,23 @@ __device__ __forceinline__ float gelu_grad_f(float x) {
   return 0.5f * (1.f + t) + 0.5f * x * (1.f - t * t) * c * (1.f + 3.f * 0.044715f * x * x);
 }
 
+// Hardware tanh approximation (about 2^-11 relative error): used where the
+// result is rounded to bf16 (2^-8) right after.
+__device__ __forceinline__ float tanh_fast(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float gelu_fast(float x) {
+  const float c = 0.7978845608028654f;
+  return 0.5f * x * (1.f + tanh_fast(c * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float gelu_grad_fast(float x) {
+  const float c = 0.7978845608028654f;
+  const float t = tanh_fast(c * (x + 0.044715f * x * x * x));
+  return 0.5f * (1.f + t) + 0.5f * x * (1.f - t * t) * c * (1.f + 3.f * 0.044715f * x * x);
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -8,10 +8,15 @@
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
 //               issues tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16),
 //               committing each stage back to the producer.
-//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns per chunk, bias /
-//               GELU / dGELU / residual in fp32, stores to global memory; the
-//               second accumulator lets tile t+1's main loop overlap tile t's
-//               epilogue.
+//   warps 2..9  epilogue (two warps per TMEM lane quadrant, each owning half of
+//               the 256 columns): tcgen05.ld 32 lanes x 32 columns, a swizzled
+//               shared-memory transpose so that every global access of the
+//               epilogue (bias, dGELU input, residual) is row-coalesced, then
+//               bias / GELU / dGELU / residual in fp32; outputs are written back
+//               into the warp's buffer as a dense tile and leave with one TMA
+//               bulk tensor store (reduce-add for fp32 accumulation) per output;
+//               the second accumulator lets tile t+1's main loop overlap tile
+//               t's epilogue.
 // Every mbarrier wait is bounded (about one second): on expiry the CTA records
 // DEV_ERR_TIMEOUT in the device error word, drains its in-flight copies and
 // MMAs, frees TMEM and returns.
@@ -34,8 +39,10 @@ constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KB
 constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr int TC_MN_CHUNK_BYTES = 64 * TC_BK * 2;  // one 64-wide MN chunk of an MN-major tile
 constexpr int TC_BAR_BYTES = 256;
-constexpr int TC_SMEM = TC_STAGES * TC_STAGE_BYTES + 1024 + TC_BAR_BYTES;
-constexpr int TC_THREADS = 192;
+constexpr int TC_EPI_WARPS = 8;
+constexpr int TC_EPI_STAGE_BYTES = 32 * 32 * 4;  // one 32x32 fp32 chunk per epilogue warp
+constexpr int TC_SMEM = TC_STAGES * TC_STAGE_BYTES + TC_EPI_WARPS * TC_EPI_STAGE_BYTES + 1024 + TC_BAR_BYTES;
+constexpr int TC_THREADS = 64 + 32 * TC_EPI_WARPS;
 constexpr uint64_t TC_WAIT_NS = 1000000000ull;  // bounded waits: 1 s
 
 struct TcGroup {
@@ -44,11 +51,16 @@ struct TcGroup {
   int amap[2], bmap[2];
   int a_mn, b_mn;
   uint32_t idesc;
+  // Output path: TMA bulk tensor stores of 32x32 chunks staged in shared
+  // memory (out_tma), else per-thread stores.  omap / omap2: maps of `out`
+  // and of the GELU output; out_accum: TMA reduce-add into fp32 `out`.
+  int out_tma, out_f32, out_accum, omap, omap2;
+  int kind;  // EpiKind specialisation used by the epilogue
   EpiParams epi;
 };
 
 struct TcParams {
-  CUtensorMap maps[8];
+  CUtensorMap maps[12];
   TcGroup grp[2];
   int ngroups, total_tiles;
   int* err;
@@ -129,6 +141,185 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
         "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])                                            \
       : "r"(taddr))
 
+
+// ---- CTA-pair (cta_group::2) helpers
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cluster address of the same shared variable in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > TC_WAIT_NS) { *abort_flag = 1; return false; }
+  }
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// TMA load into this CTA's shared memory, completing bytes on an mbarrier that
+// may live in the peer CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void tc_mma_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+// Arrive on the barrier at the same offset in both CTAs of the pair once this
+// thread's earlier MMAs are complete.
+__device__ __forceinline__ void tc_commit_pair_both(uint32_t bar) {
+  const uint16_t mask = 0x3;
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+               "h"(mask)
+               : "memory");
+}
+__device__ __forceinline__ void tc_commit_pair_local(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+// ---- TMA bulk stores from shared memory
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// One epilogue warp's 32x32 accumulator chunk (rows row0.., columns col0..),
+// already loaded from TMEM into r (lane = row).  The chunk is transposed
+// through the warp's 4 KB shared buffer so that the epilogue's global reads are
+// row-coalesced; results go out either as one TMA bulk tensor store per output
+// (written back into the same buffer as a dense row-major tile) or, when the
+// output cannot be described by a tensor map, as coalesced per-thread stores.
+// KIND fixes at compile time which inputs the epilogue reads; everything the
+// chunk needs arrives by value so that it stays in registers.
+struct EpiOut {
+  int M, N, out_tma, out_f32, out_accum, omap, omap2, gelu;
+};
+
+template <typename act_t, int KIND>
+__device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep, const EpiIn q, const EpiOut o,
+                                          float4* stage, uint32_t stage_s, int lane, int row0, int col0,
+                                          const uint32_t* r) {
+  if (o.out_tma) {  // the previous chunk's TMA stores must have read this buffer
+    if (lane == 0) bulk_wait_read_all();
+    __syncwarp();
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    stage[lane * 8 + (j ^ (lane & 7))] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                                     __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+  __syncwarp();
+  const int rb = lane >> 3, ch = lane & 7;
+  if (!o.out_tma) {
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      const int rr = it * 4 + rb;
+      float4 v4 = stage[rr * 8 + (ch ^ (rr & 7))];
+      float v[4] = {v4.x, v4.y, v4.z, v4.w};
+      epi_row<act_t, 4>(*ep, o.M, o.N, row0 + rr, col0 + ch * 4, v);
+    }
+    __syncwarp();
+    return;
+  }
+  float4 y[8];
+#pragma unroll
+  for (int it = 0; it < 8; ++it) {
+    const int rr = it * 4 + rb;
+    y[it] = epi_value4<act_t, KIND>(q, o.M, o.N, row0 + rr, col0 + ch * 4, stage[rr * 8 + (ch ^ (rr & 7))]);
+  }
+  __syncwarp();
+  const bool gelu = (KIND & EK_GELU) && (KIND != EK_ANY || o.gelu);
+  if (o.out_f32) {
+    float* so = reinterpret_cast<float*>(stage);
+#pragma unroll
+    for (int it = 0; it < 8; ++it) store4(so + (it * 4 + rb) * 32 + ch * 4, y[it]);
+  } else {
+    act_t* so = reinterpret_cast<act_t*>(stage);
+#pragma unroll
+    for (int it = 0; it < 8; ++it) store4(so + (it * 4 + rb) * 32 + ch * 4, y[it]);
+    if (gelu) {
+#pragma unroll
+      for (int it = 0; it < 8; ++it)
+        store4(so + 1024 + (it * 4 + rb) * 32 + ch * 4,
+               make_float4(epi_gelu<act_t>(y[it].x), epi_gelu<act_t>(y[it].y), epi_gelu<act_t>(y[it].z),
+                           epi_gelu<act_t>(y[it].w)));
+    }
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    if (o.out_accum) tma_reduce_add_2d(&p.maps[o.omap], stage_s, col0, row0);
+    else tma_store_2d(&p.maps[o.omap], stage_s, col0, row0);
+    if (gelu) tma_store_2d(&p.maps[o.omap2], stage_s + 2048, col0, row0);
+    bulk_commit();
+  }
+}
+
+// Runs one chunk with the specialisation the group was prepared for.
+template <typename act_t>
+__device__ __forceinline__ void epi_chunk_dispatch(int kind, const TcParams& p, const EpiParams* ep, const EpiIn q,
+                                                   const EpiOut o, float4* stage, uint32_t stage_s, int lane, int row0,
+                                                   int col0, const uint32_t* r) {
+  switch (kind) {
+    case 0: epi_chunk<act_t, 0>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_BIAS: epi_chunk<act_t, EK_BIAS>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_BIAS | EK_GELU: epi_chunk<act_t, EK_BIAS | EK_GELU>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_DGELU: epi_chunk<act_t, EK_DGELU>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_BIAS | EK_RESID: epi_chunk<act_t, EK_BIAS | EK_RESID>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_BIAS | EK_BIAS2 | EK_RESID:
+      epi_chunk<act_t, EK_BIAS | EK_BIAS2 | EK_RESID>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    default: epi_chunk<act_t, EK_ANY>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+  }
+}
+
+__device__ __forceinline__ EpiOut epi_out_of(const TcGroup& G) {
+  EpiOut o;
+  o.M = G.M; o.N = G.N; o.out_tma = G.out_tma; o.out_f32 = G.out_f32; o.out_accum = G.out_accum;
+  o.omap = G.omap; o.omap2 = G.omap2; o.gelu = G.epi.op == EPI_GELU;
+  return o;
+}
+
 __device__ __forceinline__ void decode_tile(const TcParams& p, int tile, int& g, int& m0, int& n0) {
   g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
   const TcGroup& G = p.grp[g];
@@ -142,7 +333,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t bar_base = base + TC_STAGES * TC_STAGE_BYTES;
+  const uint32_t epi_base = base + TC_STAGES * TC_STAGE_BYTES;
+  const uint32_t bar_base = epi_base + TC_EPI_WARPS * TC_EPI_STAGE_BYTES;
   uint8_t* bar_ptr = smem_raw + (bar_base - raw);
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
   auto empty_bar = [&](int s) { return bar_base + 8u * (TC_STAGES + s); };
@@ -155,7 +347,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   if (threadIdx.x == 0) {
     for (int s = 0; s < TC_STAGES; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
+    for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), TC_EPI_WARPS); }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -273,34 +465,39 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < TC_WAIT_NS) {}
     }
   } else {
-    // ------------------------------------------------ epilogue (warps 2..5)
-    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    // ------------------------------------------------ epilogue (warps 2..9)
+    const int q = warp & 3;             // TMEM lane quadrant this warp may access
+    const int half = (warp - 2) >> 2;   // which 128 of the 256 accumulator columns
+    const uint32_t stage_s = epi_base + (warp - 2) * TC_EPI_STAGE_BYTES;
+    float4* stage = reinterpret_cast<float4*>(smem_raw + (stage_s - raw));
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < p.total_tiles; tile += gridDim.x) {
       int g, m0, n0;
       decode_tile(p, tile, g, m0, n0);
       const TcGroup& G = p.grp[g];
+      const EpiOut eo = epi_out_of(G);
+      const EpiIn ei = epi_in(G.epi);
+      const int kind = G.kind;
       if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag)) break;
       tc_fence_after();
-      const int row = m0 + q * 32 + lane;
-      for (int c = 0; c < TC_BN / 32; ++c) {
-        const int col0 = n0 + c * 32;
-        if (col0 >= G.N) break;
+      for (int c = 0; c < TC_BN / 64; ++c) {
+        const int col0 = n0 + half * (TC_BN / 2) + c * 32;
+        if (col0 >= eo.N) break;
         uint32_t r[32];
-        const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + c * 32);
+        const uint32_t taddr =
+            tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2) + c * 32);
         TMEM_LD32(taddr, r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-        float v[32];
-#pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-        epi_row<act_t, 32>(G.epi, G.M, G.N, row, col0, v);
+        epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, m0 + q * 32, col0, r);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -308,6 +505,224 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
+  }
+}
+
+
+// ------------------------------------------------------------ CTA-pair kernel
+// Same contract as gemm_tc_kernel, but a cluster of two CTAs (two SMs) computes
+// a 256x256 output tile with tcgen05.mma.cta_group::2 (M=256, N=256, K=16):
+// each CTA stages its own 128 rows of A and 128 of the 256 B rows, so every SM
+// moves 32 KB per 64-deep K step instead of 48 KB and keeps six stages in
+// flight.  The even CTA issues the MMAs; its full barriers collect both CTAs'
+// TMA bytes; commits arrive on both CTAs' barriers; each CTA's epilogue reads
+// its own 128 accumulator rows from its TMEM.
+constexpr int T2_STAGES = 6;
+constexpr int T2_A_BYTES = 128 * TC_BK * 2;  // 16 KB: this CTA's 128 rows of A
+constexpr int T2_B_BYTES = 128 * TC_BK * 2;  // 16 KB: this CTA's 128 rows of B
+constexpr int T2_STAGE_BYTES = T2_A_BYTES + T2_B_BYTES;
+constexpr int T2_SMEM = T2_STAGES * T2_STAGE_BYTES + TC_EPI_WARPS * TC_EPI_STAGE_BYTES + 1024 + TC_BAR_BYTES;
+constexpr int T2_TILE = 256;
+
+__device__ __forceinline__ void decode_tile2(const TcParams& p, int tile, int& g, int& m0, int& n0) {
+  g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+  const TcGroup& G = p.grp[g];
+  const int local = tile - G.tile_start;
+  m0 = (local % G.m_tiles) * T2_TILE;
+  n0 = (local / G.m_tiles) * T2_TILE;
+}
+
+template <typename act_t>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
+    gemm_tc2_kernel(const __grid_constant__ TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t epi_base = base + T2_STAGES * T2_STAGE_BYTES;
+  const uint32_t bar_base = epi_base + TC_EPI_WARPS * TC_EPI_STAGE_BYTES;
+  uint8_t* bar_ptr = smem_raw + (bar_base - raw);
+  auto full_bar = [&](int s) { return bar_base + 8u * s; };
+  auto empty_bar = [&](int s) { return bar_base + 8u * (T2_STAGES + s); };
+  auto tfull_bar = [&](int b) { return bar_base + 8u * (2 * T2_STAGES + b); };
+  auto tempty_bar = [&](int b) { return bar_base + 8u * (2 * T2_STAGES + 2 + b); };
+  const uint32_t drain_bar = bar_base + 8u * (2 * T2_STAGES + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_ptr + 8 * (2 * T2_STAGES + 5));
+  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(bar_ptr + 8 * (2 * T2_STAGES + 5) + 4);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < T2_STAGES; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+    for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 2 * TC_EPI_WARPS); }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)), "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (both CTAs)
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_mask = 0, issued_par = 0;
+    bool ok = true;
+    for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
+      int g, m0, n0;
+      decode_tile2(p, tile, g, m0, n0);
+      const TcGroup& G = p.grp[g];
+      const int arow = m0 + (int)rank * 128, brow = n0 + (int)rank * 128;
+      for (int s = 0; s < G.nseg && ok; ++s) {
+        const CUtensorMap* am = &p.maps[G.amap[s]];
+        const CUtensorMap* bm = &p.maps[G.bmap[s]];
+        for (int kb = 0; kb < G.kb[s]; ++kb) {
+          if (!mbar_wait_cluster(empty_bar(stage), phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (lane == 0) {
+            const uint32_t fb = map_to_rank(full_bar(stage), 0);
+            const uint32_t sa = base + stage * T2_STAGE_BYTES;
+            const uint32_t sb = sa + T2_A_BYTES;
+            const int k0 = kb * TC_BK;
+            if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * T2_STAGE_BYTES);
+            if (G.a_mn) {
+              tma_load_2d_pair(sa, am, arow, k0, fb);
+              tma_load_2d_pair(sa + TC_MN_CHUNK_BYTES, am, arow + 64, k0, fb);
+            } else {
+              tma_load_2d_pair(sa, am, k0, arow, fb);
+            }
+            if (G.b_mn) {
+              tma_load_2d_pair(sb, bm, brow, k0, fb);
+              tma_load_2d_pair(sb + TC_MN_CHUNK_BYTES, bm, brow + 64, k0, fb);
+            } else {
+              tma_load_2d_pair(sb, bm, k0, brow, fb);
+            }
+          }
+          __syncwarp();
+          issued_mask |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == T2_STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+    if (!ok) {
+      if (leader) {
+        // The leader's full barriers collect both CTAs' bytes: wait for every
+        // issued stage so no copy lands after shared memory is released.
+        for (int s = 0; s < T2_STAGES; ++s) {
+          if (!(issued_mask & (1u << s))) continue;
+          const uint32_t par = (issued_par >> s) & 1u;
+          const uint64_t t0 = global_timer_ns();
+          while (!mbar_try_wait_cluster(full_bar(s), par) && global_timer_ns() - t0 < TC_WAIT_NS) {}
+        }
+      }
+      if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (even CTA only)
+    if (leader) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true, issued_any = false;
+      for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
+        int g, m0, n0;
+        decode_tile2(p, tile, g, m0, n0);
+        const TcGroup& G = p.grp[g];
+        if (!mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * TC_BN;
+        uint32_t accum = 0;
+        for (int s = 0; s < G.nseg && ok; ++s) {
+          for (int kb = 0; kb < G.kb[s]; ++kb) {
+            if (!mbar_wait_cluster(full_bar(stage), phase, abort_flag)) { ok = false; break; }
+            tc_fence_after();
+            if (lane == 0) {
+              const uint32_t sa = base + stage * T2_STAGE_BYTES;
+              const uint32_t sb = sa + T2_A_BYTES;
+#pragma unroll
+              for (int k = 0; k < TC_BK / 16; ++k) {
+                const uint64_t ad = G.a_mn ? smem_desc(sa + k * 2048, TC_MN_CHUNK_BYTES, 1024)
+                                           : smem_desc(sa + k * 32, 16, 1024);
+                const uint64_t bd = G.b_mn ? smem_desc(sb + k * 2048, TC_MN_CHUNK_BYTES, 1024)
+                                           : smem_desc(sb + k * 32, 16, 1024);
+                tc_mma_pair(d_tmem, ad, bd, G.idesc, accum);
+                accum = 1;
+              }
+              tc_commit_pair_both(empty_bar(stage));
+            }
+            __syncwarp();
+            issued_any = true;
+            if (++stage == T2_STAGES) { stage = 0; phase ^= 1u; }
+          }
+        }
+        if (!ok) break;
+        if (lane == 0) tc_commit_pair_both(tfull_bar(acc));
+        __syncwarp();
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      }
+      if (!ok && issued_any) {
+        if (lane == 0) tc_commit_pair_local(drain_bar);
+        __syncwarp();
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < TC_WAIT_NS) {}
+      }
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 2..9, both CTAs)
+    const int q = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const uint32_t stage_s = epi_base + (warp - 2) * TC_EPI_STAGE_BYTES;
+    float4* stage = reinterpret_cast<float4*>(smem_raw + (stage_s - raw));
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = cluster_id; tile < p.total_tiles; tile += nclusters) {
+      int g, m0, n0;
+      decode_tile2(p, tile, g, m0, n0);
+      const TcGroup& G = p.grp[g];
+      const EpiOut eo = epi_out_of(G);
+      const EpiIn ei = epi_in(G.epi);
+      const int kind = G.kind;
+      if (!mbar_wait_cluster(tfull_bar(acc), acc_phase, abort_flag)) break;
+      tc_fence_after();
+      const int row0 = m0 + (int)rank * 128 + q * 32;
+      for (int c = 0; c < TC_BN / 64; ++c) {
+        const int col0 = n0 + half * (TC_BN / 2) + c * 32;
+        if (col0 >= eo.N) break;
+        uint32_t r[32];
+        const uint32_t taddr =
+            tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2) + c * 32);
+        TMEM_LD32(taddr, r);
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, row0, col0, r);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(tempty_bar(acc));
+        else mbar_arrive_remote(map_to_rank(tempty_bar(acc), 0));
+      }
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
   }
 }
 
@@ -348,9 +763,24 @@ bool encode_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer,
   return true;
 }
 
+// 2-D map for the epilogue's TMA stores: 32x32 boxes, no swizzle.  Returns
+// false (no error) when the output cannot be described by a tensor map; the
+// kernel then stores with plain per-thread instructions.
+bool encode_out_map(CUtensorMap* m, const void* ptr, int f32, uint64_t cols, uint64_t rows, uint64_t ld) {
+  const uint64_t esz = f32 ? 4 : 2;
+  if (!ptr || (reinterpret_cast<uintptr_t>(ptr) & 15) || ((ld * esz) & 15)) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * esz};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr),
+                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B,
 // A/B major-ness, N>>3 at bits 17-22, M>>4 at bits 24-28.
-uint32_t make_idesc(int a_mn, int b_mn) {
+uint32_t make_idesc(int a_mn, int b_mn, int m) {
   uint32_t d = 0;
   d |= 1u << 4;             // D format: f32
   d |= 1u << 7;             // A format: bf16
@@ -358,7 +788,7 @@ uint32_t make_idesc(int a_mn, int b_mn) {
   d |= (uint32_t)a_mn << 15;
   d |= (uint32_t)b_mn << 16;
   d |= (uint32_t)(TC_BN >> 3) << 17;
-  d |= (uint32_t)(TC_BM >> 4) << 24;
+  d |= (uint32_t)(m >> 4) << 24;
   return d;
 }
 
@@ -384,13 +814,37 @@ int num_sms() {
 }
 
 int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg) {
+  return gemm_tc_engine(c, 0, dev_err, s, msg);
+}
+
+int gemm_tc_engine(const GemmCall& c, int pair, int* dev_err, cudaStream_t s, std::string* msg) {
   if (!get_encoder(msg)) return 4;
   static bool attr_set = false;
+  static int pair_clusters = 0;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(gemm_tc2_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, T2_SMEM);
     if (e != cudaSuccess) { if (msg) *msg = std::string("gemm_tc smem attribute: ") + cudaGetErrorString(e); return 4; }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (num_sms() / 2), 1, 1);
+    cfg.blockDim = dim3(TC_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = T2_SMEM;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 2; attr.val.clusterDim.y = 1; attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<bf16>, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = num_sms() / 2;
+    }
+    pair_clusters = n;
     attr_set = true;
   }
+  const int bm = pair ? T2_TILE : TC_BM, bn = pair ? T2_TILE : TC_BN;
+  const int a_rows = 128, b_rows = pair ? 128 : TC_BN;  // K-major TMA box heights per CTA
   TcParams p;
   memset(&p, 0, sizeof(p));
   int nmaps = 0, tiles = 0;
@@ -399,8 +853,8 @@ int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg) {
     const GemmGroupDesc& G = c.g[g];
     TcGroup& T = p.grp[g];
     T.M = G.M; T.N = G.N; T.nseg = G.nseg;
-    T.m_tiles = (G.M + TC_BM - 1) / TC_BM;
-    T.n_tiles = (G.N + TC_BN - 1) / TC_BN;
+    T.m_tiles = (G.M + bm - 1) / bm;
+    T.n_tiles = (G.N + bn - 1) / bn;
     T.tile_start = tiles;
     T.epi = G.epi;
     const EpiParams& e = G.epi;
@@ -423,24 +877,52 @@ int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg) {
       if (S.A.mn_major) {
         if (!encode_map(&p.maps[nmaps], S.A.ptr, G.M, S.K, S.A.ld, 64, TC_BK, msg)) return 1;
       } else {
-        if (!encode_map(&p.maps[nmaps], S.A.ptr, S.K, G.M, S.A.ld, TC_BK, TC_BM, msg)) return 1;
+        if (!encode_map(&p.maps[nmaps], S.A.ptr, S.K, G.M, S.A.ld, TC_BK, a_rows, msg)) return 1;
       }
       T.amap[sg] = nmaps++;
       if (S.B.mn_major) {
         if (!encode_map(&p.maps[nmaps], S.B.ptr, G.N, S.K, S.B.ld, 64, TC_BK, msg)) return 1;
       } else {
-        if (!encode_map(&p.maps[nmaps], S.B.ptr, S.K, G.N, S.B.ld, TC_BK, TC_BN, msg)) return 1;
+        if (!encode_map(&p.maps[nmaps], S.B.ptr, S.K, G.N, S.B.ld, TC_BK, b_rows, msg)) return 1;
       }
       T.bmap[sg] = nmaps++;
     }
-    T.idesc = make_idesc(T.a_mn, T.b_mn);
+    T.idesc = make_idesc(T.a_mn, T.b_mn, pair ? 256 : TC_BM);
+    // output maps (TMA stores) when every output of the group allows them
+    {
+      const int k = epi_kind(e);
+      const bool special = k == 0 || k == EK_BIAS || k == (EK_BIAS | EK_GELU) || k == EK_DGELU ||
+                           k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID);
+      T.kind = special ? k : EK_ANY;
+    }
+    T.out_f32 = e.out_mode != OUT_ACT && e.op != EPI_GELU;
+    T.out_accum = e.out_mode == OUT_F32_ACCUM;
+    T.out_tma = 0;
+    T.omap = T.omap2 = 0;
+    if (nmaps + 2 <= 12 && encode_out_map(&p.maps[nmaps], e.out, T.out_f32, G.N, G.M, e.ldo)) {
+      T.omap = nmaps;
+      bool ok = true;
+      if (e.op == EPI_GELU) {
+        ok = encode_out_map(&p.maps[nmaps + 1], e.out2, 0, G.N, G.M, e.ldo2);
+        T.omap2 = nmaps + 1;
+      }
+      if (ok) {
+        T.out_tma = 1;
+        nmaps += (e.op == EPI_GELU) ? 2 : 1;
+      }
+    }
     tiles += T.m_tiles * T.n_tiles;
   }
   p.total_tiles = tiles;
   p.err = dev_err;
   if (tiles == 0) return 0;
-  const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<bf16><<<grid, TC_THREADS, TC_SMEM, s>>>(p);
+  if (pair) {
+    const int clusters = tiles < pair_clusters ? tiles : pair_clusters;
+    gemm_tc2_kernel<bf16><<<2 * clusters, TC_THREADS, T2_SMEM, s>>>(p);
+  } else {
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    gemm_tc_kernel<bf16><<<grid, TC_THREADS, TC_SMEM, s>>>(p);
+  }
   count_launches(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) { if (msg) *msg = std::string("gemm_tc launch: ") + cudaGetErrorString(e); return 4; }

@@ -23,12 +23,14 @@ def _dev_bf16(a, ld_mult=8):
     return t.cuda()
 
 
-SHAPES = [(128, 256, 64), (256, 512, 1024), (300, 520, 200), (1, 17, 8), (129, 257, 65), (640, 1000, 768)]
+SHAPES = [(128, 256, 64), (256, 512, 1024), (300, 520, 200), (1, 17, 8), (129, 257, 65), (640, 1000, 768),
+          (2048, 2304, 512)]  # the last spans more 256x256 tiles than there are CTA pairs on the GPU
 
 
+@pytest.mark.parametrize("engine", ["tcgen05", "tcgen05_pair"])
 @pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (0, 1), (1, 0), (1, 1)])
 @pytest.mark.parametrize("M,N,K", SHAPES)
-def test_gemm_tcgen05_matches_matmul(M, N, K, a_mn, b_mn):
+def test_gemm_tcgen05_matches_matmul(M, N, K, a_mn, b_mn, engine):
     import torch
     from paper_2510_14614_gb300 import fal
     rng = np.random.default_rng(M * 7 + N * 3 + K + 11 * a_mn + 13 * b_mn)
@@ -40,7 +42,7 @@ def test_gemm_tcgen05_matches_matmul(M, N, K, a_mn, b_mn):
     Bt = _dev_bf16(B.T if b_mn else B)
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
     C = fal.gemm(At, Bt, M, N, K, a_mn_major=a_mn, b_mn_major=b_mn, bias=torch.as_tensor(bias).cuda(),
-                 out_f32=True, engine="tcgen05", err=err, ldc=(N + 7) // 8 * 8)
+                 out_f32=True, engine=engine, err=err, ldc=(N + 7) // 8 * 8)
     torch.cuda.synchronize()
     assert int(err.item()) == 0
     got = C.cpu().numpy()
@@ -62,6 +64,13 @@ def test_gemm_tcgen05_bf16_output_and_simt_engine(M, N, K):
     np.testing.assert_array_equal(Cb, bf16_round(Cb))
     Cs = fal.gemm(At, Bt, M, N, K, out_f32=True, engine="simt", ldc=(N + 7) // 8 * 8).cpu().numpy()
     assert rel_fro(Cs, ref) < 2e-6
+    # a bf16 output whose row pitch is not a multiple of 16 bytes cannot be a
+    # TMA store target: the kernel falls back to per-thread stores
+    ldc = (N + 3) // 4 * 4
+    if ldc % 8 == 0:
+        ldc += 4
+    Cf = fal.gemm(At, Bt, M, N, K, out_f32=False, engine="tcgen05", ldc=ldc).float().cpu().numpy()
+    np.testing.assert_array_equal(Cf, Cb)
 
 
 @pytest.mark.parametrize("hd", [64, 128])
