@@ -1,11 +1,11 @@
 // Causal multi-head attention, forward and backward (the MHA_i of every block).
 //
-// bf16 path: flash-attention style kernels (online softmax, scores never
-// written to HBM) on warp-level bf16 MMA with fp32 accumulation.  64 query
-// rows x 64 keys per tile, 4 warps per CTA (16 rows each), K/V tiles streamed
-// through shared memory with cp.async (double-buffered in the forward).
-// Backward: one CTA per (64-key block, head); dK/dV accumulate in registers,
-// dQ accumulates in an fp32 scratch buffer with vector atomics.
+// bf16 path: the forward runs on tcgen05 (attention_tc.cu).  The backward here
+// is flash-attention style (scores recomputed, never written to HBM) on
+// warp-level bf16 MMA with fp32 accumulation: one CTA per (64-key block, head),
+// 4 warps of 16 keys, query tiles of 64 streamed through shared memory with
+// cp.async; dK/dV accumulate in registers, dQ in an fp32 scratch buffer with
+// vector atomics.
 // fp32 debug path: one thread per query row, plain fp32 arithmetic.
 //
 // Scores: S = Q K^T / sqrt(hd), key j visible to query t iff j <= t.  The
@@ -70,152 +70,6 @@ __device__ __forceinline__ void load_tile(uint32_t sbase, const bf16* g, long ld
     const bool valid = t < T;
     const bf16* src = g + ((long)b * T + (valid ? t : 0)) * ld + coff + c;
     cp_async16(sbase + tile_off<HD>(r, c), src, valid);
-  }
-}
-
-// ------------------------------------------------------------ forward (bf16)
-template <int HD>
-__global__ void __launch_bounds__(128) attn_fwd_kernel(const bf16* __restrict__ qkv, bf16* __restrict__ ctx,
-                                                       float* __restrict__ lse, int T, int H, float scale_log2) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  const uint32_t sQ = smem_addr(smem);
-  const uint32_t sK0 = sQ + 64 * HD * 2;
-  const uint32_t sV0 = sK0 + 2 * 64 * HD * 2;
-  const int nqb = (T + 63) / 64;
-  const int qb = nqb - 1 - blockIdx.x;  // heaviest blocks first
-  const int bh = blockIdx.y, b = bh / H, h = bh % H;
-  const int d = H * HD;
-  const long ld = 3L * d;
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int g = lane / 4, t4 = lane % 4;
-
-  load_tile<HD, 128>(sQ, qkv, ld, b, T, qb * 64, h * HD);
-  load_tile<HD, 128>(sK0, qkv, ld, b, T, 0, d + h * HD);
-  load_tile<HD, 128>(sV0, qkv, ld, b, T, 0, 2 * d + h * HD);
-  cp_async_commit();
-
-  uint32_t qf[HD / 16][4];
-  float o[HD / 8][4];
-#pragma unroll
-  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
-  const int qrow0 = qb * 64 + warp * 16 + g;  // this thread's rows: qrow0, qrow0 + 8
-
-  for (int j = 0; j <= qb; ++j) {
-    const int buf = j & 1;
-    if (j < qb) {
-      const uint32_t sKn = sK0 + (buf ^ 1) * 64 * HD * 2, sVn = sV0 + (buf ^ 1) * 64 * HD * 2;
-      load_tile<HD, 128>(sKn, qkv, ld, b, T, (j + 1) * 64, d + h * HD);
-      load_tile<HD, 128>(sVn, qkv, ld, b, T, (j + 1) * 64, 2 * d + h * HD);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    __syncthreads();
-    if (j == 0) {
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
-        const int r = warp * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = kk * 16 + 8 * (lane / 16);
-        ldsm_x4(sQ + tile_off<HD>(r, c), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
-      }
-    }
-    const uint32_t sK = sK0 + buf * 64 * HD * 2, sV = sV0 + buf * 64 * HD * 2;
-    float s[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-#pragma unroll
-      for (int nb = 0; nb < 8; nb += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = nb * 8 + (lane % 8) + 8 * (lane / 16);
-        const int c = kk * 16 + 8 * ((lane / 8) % 2);
-        ldsm_x4(sK + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(s[nb], qf[kk], b0, b1);
-        mma_bf16(s[nb + 1], qf[kk], b2, b3);
-      }
-    }
-    // scale, mask, online softmax
-    float mx[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = j * 64 + nb * 8 + 2 * t4 + (e & 1);
-        const int qr = qrow0 + (e >> 1) * 8;
-        float v = s[nb][e] * scale_log2;
-        if (key > qr || key >= T) v = -INFINITY;
-        s[nb][e] = v;
-        mx[e >> 1] = fmaxf(mx[e >> 1], v);
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
-    }
-    float corr[2], mnew[2], rs[2] = {0.f, 0.f};
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      mnew[r] = fmaxf(mrow[r], mx[r]);
-      corr[r] = (mrow[r] == -INFINITY) ? 0.f : exp2f(mrow[r] - mnew[r]);
-      mrow[r] = mnew[r];
-    }
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int r = e >> 1;
-        const float pv = (s[nb][e] == -INFINITY) ? 0.f : exp2f(s[nb][e] - mnew[r]);
-        s[nb][e] = pv;
-        rs[r] += pv;
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 1);
-      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 2);
-      lrow[r] = lrow[r] * corr[r] + rs[r];
-    }
-#pragma unroll
-    for (int i = 0; i < HD / 8; ++i) {
-      o[i][0] *= corr[0]; o[i][1] *= corr[0];
-      o[i][2] *= corr[1]; o[i][3] *= corr[1];
-    }
-    // O += P V
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t a[4];
-      a[0] = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
-      a[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
-      a[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-      a[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-      for (int nd = 0; nd < HD / 8; nd += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = kk * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = nd * 8 + 8 * (lane / 16);
-        ldsm_x4_t(sV + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(o[nd], a, b0, b1);
-        mma_bf16(o[nd + 1], a, b2, b3);
-      }
-    }
-    __syncthreads();
-  }
-  // normalise and store
-#pragma unroll
-  for (int r = 0; r < 2; ++r) {
-    const int t = qrow0 + r * 8;
-    if (t >= T) continue;
-    const float inv = 1.f / lrow[r];
-    bf16* out = ctx + ((long)b * T + t) * d + h * HD;
-#pragma unroll
-    for (int nd = 0; nd < HD / 8; ++nd) {
-      *reinterpret_cast<uint32_t*>(out + nd * 8 + 2 * t4) = pack_bf16(o[nd][2 * r] * inv, o[nd][2 * r + 1] * inv);
-    }
-    if (t4 == 0) lse[(long)bh * T + t] = mrow[r] + log2f(lrow[r]);
   }
 }
 
@@ -536,20 +390,6 @@ __global__ void zero_kv_grad(float* dqkv, long rows, int d) {
 }
 
 template <int HD>
-int launch_fwd(int B, int T, int H, const void* qkv, void* ctx, float* lse, cudaStream_t s) {
-  const int smem = 5 * 64 * HD * 2;
-  static bool set = false;
-  if (!set) {
-    cudaFuncSetAttribute(attn_fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    set = true;
-  }
-  dim3 grid((T + 63) / 64, B * H);
-  attn_fwd_kernel<HD><<<grid, 128, smem, s>>>(reinterpret_cast<const bf16*>(qkv), reinterpret_cast<bf16*>(ctx), lse, T,
-                                             H, LOG2E / sqrtf((float)HD));
-  return 0;
-}
-
-template <int HD>
 int launch_bwd(int B, int T, int H, const void* qkv, const void* dctx, const float* lse, const float* dvec,
                float* dq_acc, void* dqkv, cudaStream_t s) {
   const int smem = 4 * 64 * HD * 2 + 64 * 64 * 2 + 2 * 64 * 4;
@@ -576,13 +416,11 @@ int check_launch(const char* what, std::string* msg) {
 
 }  // namespace
 
-int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, cudaStream_t s,
-             std::string* msg) {
+int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
+             cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
   if (act_bf16) {
-    if (hd == 64) launch_fwd<64>(B, T, H, qkv, ctx, lse, s);
-    else if (hd == 128) launch_fwd<128>(B, T, H, qkv, ctx, lse, s);
-    else { if (msg) *msg = "bf16 attention needs head_dim 64 or 128"; return 6; }
+    return attn_fwd_tc(B, T, H, hd, qkv, ctx, lse, dev_err, s, msg);
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
     const long n = (long)B * H * T;

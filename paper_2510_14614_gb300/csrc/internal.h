@@ -48,7 +48,9 @@ int gemm_tc_engine(const GemmCall& c, int pair, int* dev_err, cudaStream_t s, st
 // ---------------------------------------------------------------- attention
 // qkv: activation [B*T, 3*H*hd] (q | k | v, head-major inside each third);
 // ctx: activation [B*T, H*hd]; lse: fp32 [B, H, T] in log2 units of the scaled scores.
-int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse,
+// bf16: tcgen05 kernel (dev_err receives DEV_ERR_TIMEOUT if a bounded wait expires);
+// fp32 debug: one thread per query row.
+int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
              cudaStream_t s, std::string* msg);
 // dq_acc: fp32 [B*T, H*hd] scratch, dvec: fp32 [B, H, T] scratch.
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
@@ -110,6 +112,16 @@ int act_to_f32(int act_bf16, size_t n, const void* src, float* dst, cudaStream_t
 int act_to_f32_2d(int act_bf16, int rows, int cols, long ld, const void* src, float* dst, cudaStream_t s);
 
 int num_sms();
+
+// 2-D TMA descriptor over a row-major matrix (inner = contiguous extent, outer =
+// rows, ld in elements), bf16 or fp32, box box_inner x box_outer, 128-byte
+// swizzle or none.  False (with a message) when the driver rejects it.
+bool tma_map_2d(void* map128, const void* ptr, int f32, unsigned long long inner, unsigned long long outer,
+                unsigned long long ld, unsigned box_inner, unsigned box_outer, int swizzle128, std::string* msg);
+
+// tcgen05 flash-attention forward (bf16, head_dim 64 or 128).
+int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
+                std::string* msg);
 
 // Process-wide count of kernel launches made by the library.
 void count_launches(long long n);

@@ -40,7 +40,7 @@ int fal_kernel_gemm(int M, int N, int K, const void* A, long lda, int a_mn_major
 int fal_kernel_attention_fwd(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, void* stream) {
   if (B < 0 || T < 0 || H <= 0 || !qkv || !ctx || !lse) return FAL_ERR_ARG;
   std::string msg;
-  return map_rc(attn_fwd(1, B, T, H, hd, qkv, ctx, lse, reinterpret_cast<cudaStream_t>(stream), &msg));
+  return map_rc(attn_fwd(1, B, T, H, hd, qkv, ctx, lse, nullptr, reinterpret_cast<cudaStream_t>(stream), &msg));
 }
 
 size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd) {

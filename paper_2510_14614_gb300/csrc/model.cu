@@ -444,7 +444,7 @@ void qkv_and_attention(Ctx& c, int i, cudaStream_t s) {
   if (!c.ok()) return;
   h->err.clear();
   ProfScope ps(h, s, 1, attn_fwd_flops(h));
-  c.check(attn_fwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, s, &h->err), "attention forward");
+  c.check(attn_fwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dev_err, s, &h->err), "attention forward");
 }
 
 void up_gemm(Ctx& c, int i, cudaStream_t s) {
