@@ -1,12 +1,9 @@
 // Causal multi-head attention, forward and backward (the MHA_i of every block).
 //
-// bf16 path: the forward runs on tcgen05 (attention_tc.cu).  The backward here
-// is flash-attention style (scores recomputed, never written to HBM) on
-// warp-level bf16 MMA with fp32 accumulation: one CTA per (64-key block, head),
-// 4 warps of 16 keys, query tiles of 64 streamed through shared memory with
-// cp.async; dK/dV accumulate in registers, dQ in an fp32 scratch buffer with
-// vector atomics.
-// fp32 debug path: one thread per query row, plain fp32 arithmetic.
+// bf16 path: the tcgen05 kernels live in attention_tc.cu; this file holds the
+// backward's pre-pass (D = rowsum(dO * O), zeroed dQ accumulator) and post-pass
+// (dQ accumulator -> bf16), the fp32 debug kernels (one thread per query row,
+// plain fp32 arithmetic) and the allocation-free backward entry point.
 //
 // Scores: S = Q K^T / sqrt(hd), key j visible to query t iff j <= t.  The
 // saved log-sum-exp is in log2 units of S*log2(e).
@@ -18,60 +15,6 @@ namespace fal {
 namespace {
 
 constexpr float LOG2E = 1.4426950408889634f;
-
-// ------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
-  const int n = valid ? 16 : 0;
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-// D(16x8) += A(16x16, row) * B(16x8, col), bf16 inputs, fp32 accumulators.
-__device__ __forceinline__ void mma_bf16(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// Tile [64 rows][HD] bf16 in shared memory, 16-byte chunks XOR-swizzled by row
-// so that ldmatrix row reads hit distinct banks.
-template <int HD>
-__device__ __forceinline__ uint32_t tile_off(int row, int col) {  // col multiple of 8
-  return (uint32_t)((row * HD + (((col >> 3) ^ (row & 7)) << 3)) * 2);
-}
-
-// Loads rows [r0, r0+64) of one head's slice (column offset coff) of a
-// row-major [B*T, ld] bf16 matrix for batch b; rows >= T are zero-filled.
-template <int HD, int NT>
-__device__ __forceinline__ void load_tile(uint32_t sbase, const bf16* g, long ld, int b, int T, int r0, int coff) {
-  constexpr int CH = HD / 8;
-  for (int i = threadIdx.x; i < 64 * CH; i += NT) {
-    const int r = i / CH, c = (i % CH) * 8;
-    const int t = r0 + r;
-    const bool valid = t < T;
-    const bf16* src = g + ((long)b * T + (valid ? t : 0)) * ld + coff + c;
-    cp_async16(sbase + tile_off<HD>(r, c), src, valid);
-  }
-}
 
 // ------------------------------------------------------------ backward (bf16)
 // D[b,h,t] = sum_c dO[t,c] * O[t,c]; also clears the dQ accumulator.
@@ -104,214 +47,6 @@ __global__ void attn_bwd_post_kernel(const float* __restrict__ dq_acc, bf16* __r
     const long e = i * 4;
     const long r = e / d, c = e % d;
     store4(dqkv + r * 3L * d + c, load4(dq_acc + e));
-  }
-}
-
-template <int HD>
-__global__ void __launch_bounds__(128) attn_bwd_kernel(const bf16* __restrict__ qkv, const bf16* __restrict__ dctx,
-                                                       const float* __restrict__ lse, const float* __restrict__ dvec,
-                                                       float* __restrict__ dq_acc, bf16* __restrict__ dqkv, int T, int H,
-                                                       float scale, float scale_log2) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  const uint32_t sK = smem_addr(smem);
-  const uint32_t sV = sK + 64 * HD * 2;
-  const uint32_t sQ = sV + 64 * HD * 2;
-  const uint32_t sdO = sQ + 64 * HD * 2;
-  const uint32_t sdS = sdO + 64 * HD * 2;  // [64 q][64 keys] bf16
-  bf16* dS_ptr = reinterpret_cast<bf16*>(smem + 4 * 64 * HD * 2);
-  float* s_lse = reinterpret_cast<float*>(smem + 4 * 64 * HD * 2 + 64 * 64 * 2);
-  float* s_d = s_lse + 64;
-
-  const int nkb = (T + 63) / 64;
-  const int kb = nkb - 1 - blockIdx.x;  // shortest work last... (longest first: kb small has most q blocks)
-  const int kblk = blockIdx.x;          // process kv block index directly for load balance below
-  (void)kb;
-  const int bh = blockIdx.y, b = bh / H, h = bh % H;
-  const int d = H * HD;
-  const long ld = 3L * d;
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int g = lane / 4, t4 = lane % 4;
-  const int key0 = kblk * 64;
-
-  load_tile<HD, 128>(sK, qkv, ld, b, T, key0, d + h * HD);
-  load_tile<HD, 128>(sV, qkv, ld, b, T, key0, 2 * d + h * HD);
-  cp_async_commit();
-
-  float dk[HD / 8][4], dv[HD / 8][4];
-#pragma unroll
-  for (int i = 0; i < HD / 8; ++i)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) dk[i][e] = dv[i][e] = 0.f;
-
-  const int nqb = (T + 63) / 64;
-  for (int qb = kblk; qb < nqb; ++qb) {
-    const int q0 = qb * 64;
-    load_tile<HD, 128>(sQ, qkv, ld, b, T, q0, h * HD);
-    load_tile<HD, 128>(sdO, dctx, d, b, T, q0, h * HD);
-    cp_async_commit();
-    if (threadIdx.x < 64) {
-      const int t = q0 + threadIdx.x;
-      s_lse[threadIdx.x] = (t < T) ? lse[(long)bh * T + t] : 0.f;
-      s_d[threadIdx.x] = (t < T) ? dvec[(long)bh * T + t] : 0.f;
-    }
-    cp_async_wait<0>();
-    __syncthreads();
-
-    // S^T (16 keys of this warp x 64 queries) = K_w Q^T
-    float st[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) st[i][0] = st[i][1] = st[i][2] = st[i][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      uint32_t a[4];
-      {
-        const int r = warp * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = kk * 16 + 8 * (lane / 16);
-        ldsm_x4(sK + tile_off<HD>(r, c), a[0], a[1], a[2], a[3]);
-      }
-#pragma unroll
-      for (int nb = 0; nb < 8; nb += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = nb * 8 + (lane % 8) + 8 * (lane / 16);
-        const int c = kk * 16 + 8 * ((lane / 8) % 2);
-        ldsm_x4(sQ + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(st[nb], a, b0, b1);
-        mma_bf16(st[nb + 1], a, b2, b3);
-      }
-    }
-    // P^T = exp2(S^T * scale_log2 - lse[q]) with causal mask (q >= key)
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = key0 + warp * 16 + g + (e >> 1) * 8;
-        const int ql = nb * 8 + 2 * t4 + (e & 1);
-        const int q = q0 + ql;
-        float pv = exp2f(st[nb][e] * scale_log2 - s_lse[ql]);
-        if (q < key || q >= T || key >= T) pv = 0.f;
-        st[nb][e] = pv;
-      }
-    }
-    // dV_w += P^T dO
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t a[4];
-      a[0] = pack_bf16(st[2 * kk][0], st[2 * kk][1]);
-      a[1] = pack_bf16(st[2 * kk][2], st[2 * kk][3]);
-      a[2] = pack_bf16(st[2 * kk + 1][0], st[2 * kk + 1][1]);
-      a[3] = pack_bf16(st[2 * kk + 1][2], st[2 * kk + 1][3]);
-#pragma unroll
-      for (int nd = 0; nd < HD / 8; nd += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = kk * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = nd * 8 + 8 * (lane / 16);
-        ldsm_x4_t(sdO + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(dv[nd], a, b0, b1);
-        mma_bf16(dv[nd + 1], a, b2, b3);
-      }
-    }
-    // dP^T = V_w dO^T
-    float dpt[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) dpt[i][0] = dpt[i][1] = dpt[i][2] = dpt[i][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      uint32_t a[4];
-      {
-        const int r = warp * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = kk * 16 + 8 * (lane / 16);
-        ldsm_x4(sV + tile_off<HD>(r, c), a[0], a[1], a[2], a[3]);
-      }
-#pragma unroll
-      for (int nb = 0; nb < 8; nb += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = nb * 8 + (lane % 8) + 8 * (lane / 16);
-        const int c = kk * 16 + 8 * ((lane / 8) % 2);
-        ldsm_x4(sdO + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(dpt[nb], a, b0, b1);
-        mma_bf16(dpt[nb + 1], a, b2, b3);
-      }
-    }
-    // dS^T = P^T * (dP^T - D[q]); stash dS (q-major) in shared memory for dQ
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int ql = nb * 8 + 2 * t4 + (e & 1);
-        const float ds = st[nb][e] * (dpt[nb][e] - s_d[ql]);
-        dpt[nb][e] = ds;
-        const int kl = warp * 16 + g + (e >> 1) * 8;
-        // element (row ql, col kl) of the [64][64] q-major tile, same swizzle as tile_off<64>
-        const uint32_t off = tile_off<64>(ql, kl & ~7) / 2 + (kl & 7);
-        dS_ptr[off] = __float2bfloat16_rn(ds);
-      }
-    }
-    // dK_w += dS^T Q
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t a[4];
-      a[0] = pack_bf16(dpt[2 * kk][0], dpt[2 * kk][1]);
-      a[1] = pack_bf16(dpt[2 * kk][2], dpt[2 * kk][3]);
-      a[2] = pack_bf16(dpt[2 * kk + 1][0], dpt[2 * kk + 1][1]);
-      a[3] = pack_bf16(dpt[2 * kk + 1][2], dpt[2 * kk + 1][3]);
-#pragma unroll
-      for (int nd = 0; nd < HD / 8; nd += 2) {
-        uint32_t b0, b1, b2, b3;
-        const int r = kk * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = nd * 8 + 8 * (lane / 16);
-        ldsm_x4_t(sQ + tile_off<HD>(r, c), b0, b1, b2, b3);
-        mma_bf16(dk[nd], a, b0, b1);
-        mma_bf16(dk[nd + 1], a, b2, b3);
-      }
-    }
-    __syncthreads();
-    // dQ (rows 16*warp.. of this q block) += dS K, accumulated in fp32 scratch
-    {
-      float dq[HD / 8][4];
-#pragma unroll
-      for (int i = 0; i < HD / 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        uint32_t a[4];
-        const int r = warp * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-        const int c = kk * 16 + 8 * (lane / 16);
-        ldsm_x4(sdS + tile_off<64>(r, c), a[0], a[1], a[2], a[3]);
-#pragma unroll
-        for (int nd = 0; nd < HD / 8; nd += 2) {
-          uint32_t b0, b1, b2, b3;
-          const int rr = kk * 16 + (lane % 8) + 8 * ((lane / 8) % 2);
-          const int cc = nd * 8 + 8 * (lane / 16);
-          ldsm_x4_t(sK + tile_off<HD>(rr, cc), b0, b1, b2, b3);
-          mma_bf16(dq[nd], a, b0, b1);
-          mma_bf16(dq[nd + 1], a, b2, b3);
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        const int q = q0 + warp * 16 + g + r * 8;
-        if (q >= T) continue;
-        float* dst = dq_acc + ((long)b * T + q) * d + h * HD;
-#pragma unroll
-        for (int nd = 0; nd < HD / 8; ++nd) {
-          atomicAdd(reinterpret_cast<float2*>(dst + nd * 8 + 2 * t4),
-                    make_float2(dq[nd][2 * r] * scale, dq[nd][2 * r + 1] * scale));
-        }
-      }
-    }
-    __syncthreads();
-  }
-  // write dK (scaled) and dV for this warp's 16 keys
-#pragma unroll
-  for (int r = 0; r < 2; ++r) {
-    const int key = key0 + warp * 16 + g + r * 8;
-    if (key >= T) continue;
-    bf16* dkp = dqkv + ((long)b * T + key) * ld + d + h * HD;
-    bf16* dvp = dqkv + ((long)b * T + key) * ld + 2 * d + h * HD;
-#pragma unroll
-    for (int nd = 0; nd < HD / 8; ++nd) {
-      *reinterpret_cast<uint32_t*>(dkp + nd * 8 + 2 * t4) = pack_bf16(dk[nd][2 * r] * scale, dk[nd][2 * r + 1] * scale);
-      *reinterpret_cast<uint32_t*>(dvp + nd * 8 + 2 * t4) = pack_bf16(dv[nd][2 * r], dv[nd][2 * r + 1]);
-    }
   }
 }
 
@@ -389,22 +124,6 @@ __global__ void zero_kv_grad(float* dqkv, long rows, int d) {
   }
 }
 
-template <int HD>
-int launch_bwd(int B, int T, int H, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-               float* dq_acc, void* dqkv, cudaStream_t s) {
-  const int smem = 4 * 64 * HD * 2 + 64 * 64 * 2 + 2 * 64 * 4;
-  static bool set = false;
-  if (!set) {
-    cudaFuncSetAttribute(attn_bwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    set = true;
-  }
-  dim3 grid((T + 63) / 64, B * H);
-  attn_bwd_kernel<HD><<<grid, 128, smem, s>>>(reinterpret_cast<const bf16*>(qkv), reinterpret_cast<const bf16*>(dctx),
-                                             lse, dvec, dq_acc, reinterpret_cast<bf16*>(dqkv), T, H,
-                                             1.f / sqrtf((float)HD), LOG2E / sqrtf((float)HD));
-  return 0;
-}
-
 int check_launch(const char* what, std::string* msg) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
@@ -433,7 +152,7 @@ int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* c
 }
 
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
-             const void* dctx, void* dqkv, float* dq_acc, float* dvec, cudaStream_t s, std::string* msg) {
+             const void* dctx, void* dqkv, float* dq_acc, float* dvec, int* dev_err, cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
   const long rows = (long)B * T;
   const int d = H * hd;
@@ -443,12 +162,12 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
     dim3 pg((H + wpb - 1) / wpb, (unsigned)rows);
     attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx),
                                                dvec, dq_acc, T, H, hd);
-    if (hd == 64) launch_bwd<64>(B, T, H, qkv, dctx, lse, dvec, dq_acc, dqkv, s);
-    else launch_bwd<128>(B, T, H, qkv, dctx, lse, dvec, dq_acc, dqkv, s);
+    const int r = attn_bwd_tc(B, T, H, hd, qkv, dctx, lse, dvec, dq_acc, dqkv, dev_err, s, msg);
+    if (r) return r;
     const long n4 = rows * d / 4;
     const int blocks = (int)((n4 + 255) / 256 < 4096 ? (n4 + 255) / 256 : 4096);
     attn_bwd_post_kernel<<<blocks, 256, 0, s>>>(dq_acc, reinterpret_cast<bf16*>(dqkv), rows, d);
-    count_launches(3);
+    count_launches(2);
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
     zero_kv_grad<<<256, 256, 0, s>>>(reinterpret_cast<float*>(dqkv), rows, d);
@@ -511,7 +230,7 @@ extern "C" int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, con
   std::string msg;
   // attn_bwd's first kernel zeroes the dQ accumulator and writes every D entry,
   // so nothing left in the shared array by an earlier call leaks into this one.
-  const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, scratch + dq_floats,
+  const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, scratch + dq_floats, nullptr,
                               reinterpret_cast<cudaStream_t>(stream), &msg);
   return r == 0 ? FAL_OK : r == 1 ? FAL_ERR_ARG : r == 6 ? FAL_ERR_UNSUPPORTED : FAL_ERR_CUDA;
 }

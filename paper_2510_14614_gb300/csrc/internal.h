@@ -54,7 +54,7 @@ int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* c
              cudaStream_t s, std::string* msg);
 // dq_acc: fp32 [B*T, H*hd] scratch, dvec: fp32 [B, H, T] scratch.
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
-             const float* lse, const void* dctx, void* dqkv, float* dq_acc, float* dvec,
+             const float* lse, const void* dctx, void* dqkv, float* dq_acc, float* dvec, int* dev_err,
              cudaStream_t s, std::string* msg);
 
 // ---------------------------------------------------------------- elementwise
@@ -119,9 +119,12 @@ int num_sms();
 bool tma_map_2d(void* map128, const void* ptr, int f32, unsigned long long inner, unsigned long long outer,
                 unsigned long long ld, unsigned box_inner, unsigned box_outer, int swizzle128, std::string* msg);
 
-// tcgen05 flash-attention forward (bf16, head_dim 64 or 128).
+// tcgen05 flash-attention forward and backward main kernel (bf16, head_dim 64
+// or 128).  The backward expects dvec = rowsum(dO * O) and a zeroed dq_acc.
 int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
                 std::string* msg);
+int attn_bwd_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
+                float* dq_acc, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
 
 // Process-wide count of kernel launches made by the library.
 void count_launches(long long n);

@@ -53,7 +53,8 @@ int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const
   std::string msg;
   float* dq_acc = scratch;
   float* dvec = scratch + (size_t)B * T * H * hd;
-  return map_rc(attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, dq_acc, dvec, reinterpret_cast<cudaStream_t>(stream),
+  return map_rc(attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, dq_acc, dvec, nullptr,
+                         reinterpret_cast<cudaStream_t>(stream),
                          &msg));
 }
 

@@ -593,7 +593,8 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   if (!c.ok()) return;
   h->err.clear();
   ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h));
-  c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dq_acc, h->dvec, s, &h->err),
+  c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dq_acc, h->dvec,
+                   h->dev_err, s, &h->err),
           "attention backward");
   gemm(c, call1(BT, d, dgrad_seg(h, h->dqkv, 3 * d, p.w_qkv, d), epi_out(h->dU, d, OUT_F32)), s, "QKV dgrad");
   gemm(c, call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), epi_out(Gp(h, p.w_qkv), d, OUT_F32)), s, "QKV wgrad");
