@@ -70,13 +70,15 @@ struct TcParams {
 
 
 // One epilogue warp's 32x32 accumulator chunk (rows row0.., columns col0..),
-// already loaded from TMEM into r (lane = row).  The chunk is transposed
-// through the warp's 4 KB shared buffer so that the epilogue's global reads are
-// row-coalesced; results go out either as one TMA bulk tensor store per output
-// (written back into the same buffer as a dense row-major tile) or, when the
-// output cannot be described by a tensor map, as coalesced per-thread stores.
-// KIND fixes at compile time which inputs the epilogue reads; everything the
-// chunk needs arrives by value so that it stays in registers.
+// already loaded from TMEM into r (lane = row).  When every output of the group
+// is a TMA target (the usual case) the lane keeps its row: bias / GELU / dGELU /
+// residual are applied in registers and the row is written into the warp's
+// 4 KB buffer in the swizzled layout of the output's tensor map (64-byte rows
+// in bf16, 128-byte rows in fp32, conflict-free), then one TMA bulk tensor store
+// (reduce-add for fp32 accumulation) per output leaves the SM.  Otherwise the
+// chunk is transposed through the buffer and stored with coalesced per-thread
+// stores.  KIND fixes at compile time which inputs the epilogue reads;
+// everything the chunk needs arrives by value so that it stays in registers.
 struct EpiOut {
   int M, N, out_tma, out_f32, out_accum, omap, omap2, gelu;
 };
@@ -85,17 +87,13 @@ template <typename act_t, int KIND>
 __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep, const EpiIn q, const EpiOut o,
                                           float4* stage, uint32_t stage_s, int lane, int row0, int col0,
                                           const uint32_t* r) {
-  if (o.out_tma) {  // the previous chunk's TMA stores must have read this buffer
-    if (lane == 0) bulk_wait_read_all();
-    __syncwarp();
-  }
-#pragma unroll
-  for (int j = 0; j < 8; ++j)
-    stage[lane * 8 + (j ^ (lane & 7))] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
-                                                     __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
-  __syncwarp();
-  const int rb = lane >> 3, ch = lane & 7;
   if (!o.out_tma) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      stage[lane * 8 + (j ^ (lane & 7))] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                                       __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+    __syncwarp();
+    const int rb = lane >> 3, ch = lane & 7;
 #pragma unroll
     for (int it = 0; it < 8; ++it) {
       const int rr = it * 4 + rb;
@@ -106,28 +104,45 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep
     __syncwarp();
     return;
   }
+  // the previous chunk's TMA stores must have read this buffer
+  if (lane == 0) bulk_wait_read_all();
+  __syncwarp();
+  const int row = row0 + lane;
   float4 y[8];
 #pragma unroll
-  for (int it = 0; it < 8; ++it) {
-    const int rr = it * 4 + rb;
-    y[it] = epi_value4<act_t, KIND>(q, o.M, o.N, row0 + rr, col0 + ch * 4, stage[rr * 8 + (ch ^ (rr & 7))]);
-  }
-  __syncwarp();
+  for (int g = 0; g < 8; ++g)
+    y[g] = epi_value4<act_t, KIND>(q, o.M, o.N, row, col0 + 4 * g,
+                                   make_float4(__uint_as_float(r[4 * g]), __uint_as_float(r[4 * g + 1]),
+                                               __uint_as_float(r[4 * g + 2]), __uint_as_float(r[4 * g + 3])));
+  uint8_t* sb = reinterpret_cast<uint8_t*>(stage);
   const bool gelu = (KIND & EK_GELU) && (KIND != EK_ANY || o.gelu);
   if (o.out_f32) {
-    float* so = reinterpret_cast<float*>(stage);
 #pragma unroll
-    for (int it = 0; it < 8; ++it) store4(so + (it * 4 + rb) * 32 + ch * 4, y[it]);
+    for (int g = 0; g < 8; ++g) *reinterpret_cast<float4*>(sb + lane * 128 + ((g ^ (lane & 7)) << 4)) = y[g];
   } else {
-    act_t* so = reinterpret_cast<act_t*>(stage);
+    const int sw = (lane >> 1) & 3;
 #pragma unroll
-    for (int it = 0; it < 8; ++it) store4(so + (it * 4 + rb) * 32 + ch * 4, y[it]);
+    for (int g = 0; g < 4; ++g) {
+      uint4 pk;
+      __nv_bfloat162 t0 = __floats2bfloat162_rn(y[2 * g].x, y[2 * g].y), t1 = __floats2bfloat162_rn(y[2 * g].z, y[2 * g].w);
+      __nv_bfloat162 t2 = __floats2bfloat162_rn(y[2 * g + 1].x, y[2 * g + 1].y);
+      __nv_bfloat162 t3 = __floats2bfloat162_rn(y[2 * g + 1].z, y[2 * g + 1].w);
+      pk.x = *reinterpret_cast<uint32_t*>(&t0); pk.y = *reinterpret_cast<uint32_t*>(&t1);
+      pk.z = *reinterpret_cast<uint32_t*>(&t2); pk.w = *reinterpret_cast<uint32_t*>(&t3);
+      *reinterpret_cast<uint4*>(sb + lane * 64 + ((g ^ sw) << 4)) = pk;
+    }
     if (gelu) {
 #pragma unroll
-      for (int it = 0; it < 8; ++it)
-        store4(so + 1024 + (it * 4 + rb) * 32 + ch * 4,
-               make_float4(epi_gelu<act_t>(y[it].x), epi_gelu<act_t>(y[it].y), epi_gelu<act_t>(y[it].z),
-                           epi_gelu<act_t>(y[it].w)));
+      for (int g = 0; g < 4; ++g) {
+        uint4 pk;
+        __nv_bfloat162 t0 = __floats2bfloat162_rn(epi_gelu<act_t>(y[2 * g].x), epi_gelu<act_t>(y[2 * g].y));
+        __nv_bfloat162 t1 = __floats2bfloat162_rn(epi_gelu<act_t>(y[2 * g].z), epi_gelu<act_t>(y[2 * g].w));
+        __nv_bfloat162 t2 = __floats2bfloat162_rn(epi_gelu<act_t>(y[2 * g + 1].x), epi_gelu<act_t>(y[2 * g + 1].y));
+        __nv_bfloat162 t3 = __floats2bfloat162_rn(epi_gelu<act_t>(y[2 * g + 1].z), epi_gelu<act_t>(y[2 * g + 1].w));
+        pk.x = *reinterpret_cast<uint32_t*>(&t0); pk.y = *reinterpret_cast<uint32_t*>(&t1);
+        pk.z = *reinterpret_cast<uint32_t*>(&t2); pk.w = *reinterpret_cast<uint32_t*>(&t3);
+        *reinterpret_cast<uint4*>(sb + 2048 + lane * 64 + ((g ^ sw) << 4)) = pk;
+      }
     }
   }
   fence_proxy_async_smem();
@@ -607,9 +622,11 @@ bool encode_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer,
   return true;
 }
 
-// 2-D map for the epilogue's TMA stores: 32x32 boxes, no swizzle.  Returns
-// false (no error) when the output cannot be described by a tensor map; the
-// kernel then stores with plain per-thread instructions.
+// 2-D map for the epilogue's TMA stores: 32x32 boxes whose rows (64 B in bf16,
+// 128 B in fp32) are swizzled in shared memory (64-byte / 128-byte swizzle) so
+// that each lane can write its own row without bank conflicts.  Returns false
+// (no error) when the output cannot be described by a tensor map; the kernel
+// then stores with plain per-thread instructions.
 bool encode_out_map(CUtensorMap* m, const void* ptr, int f32, uint64_t cols, uint64_t rows, uint64_t ld) {
   const uint64_t esz = f32 ? 4 : 2;
   if (!ptr || (reinterpret_cast<uintptr_t>(ptr) & 15) || ((ld * esz) & 15)) return false;
@@ -618,8 +635,9 @@ bool encode_out_map(CUtensorMap* m, const void* ptr, int f32, uint64_t cols, uin
   cuuint32_t box[2] = {32, 32};
   cuuint32_t estr[2] = {1, 1};
   return g_encode(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr),
-                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B,
