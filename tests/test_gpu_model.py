@@ -136,6 +136,28 @@ def test_call_order_errors():
     assert e.value.code == fal.FAL_ERR_STATE
 
 
+@pytest.mark.parametrize("variant,schedule", [("fal", "two_stream"), ("gpt", "serial"), ("falplus", "serial")])
+def test_fused_train_step_matches_separate_calls(variant, schedule):
+    """fal_train_step (one call for forward, backward and AdamW) leaves the
+    same parameters as forward + backward + step called one by one (up to the
+    reduction order of atomics in the gradients)."""
+    s = SMALL
+    params = synth.perturb_params(synth.init_params(variant, s, 3), 3)
+    tok, tgt = synth.make_tokens(s, 3)
+    a, b = _model(variant, s, schedule), _model(variant, s, schedule)
+    a.set_params(params)
+    b.set_params(params)
+    for _ in range(2):
+        la = a.train_step(tok, tgt)
+        lb = b.forward(tok, tgt)
+        b.backward()
+        b.step()
+        assert abs(la - lb) <= 1e-6 * abs(lb)
+    pa, pb = a.params(), b.params()
+    for k in params:
+        np.testing.assert_allclose(pa[k], pb[k], rtol=1e-5, atol=1e-7, err_msg=k)
+
+
 def test_training_reduces_loss():
     s = SMALL
     from paper_2510_14614_gb300 import fal
