@@ -274,55 +274,56 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer
-    int stage = 0;
-    uint32_t phase = 0;
-    int acc = 0;
-    uint32_t acc_phase = 0;
-    bool ok = true, issued_any = false;
-    for (int tile = blockIdx.x; tile < p.total_tiles && ok; tile += gridDim.x) {
-      int g, m0, n0;
-      decode_tile(p, tile, g, m0, n0);
-      const TcGroup& G = p.grp[g];
-      if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
-      tc_fence_after();
-      const uint32_t d_tmem = tmem_base + acc * TC_BN;
-      uint32_t accum = 0;
-      for (int s = 0; s < G.nseg && ok; ++s) {
-        for (int kb = 0; kb < G.kb[s]; ++kb) {
+    // ------------------------------------------------ MMA issuer (one thread)
+    // The tensor pipe accepts only a few MMAs ahead, so the issuing thread
+    // blocks inside each stage's MMAs and must come back for the next stage
+    // before the queued work drains: everything per tile is hoisted into
+    // registers and the per-stage path is wait / fence / 4 MMAs / commit.
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true, issued_any = false;
+      for (int tile = blockIdx.x; tile < p.total_tiles && ok; tile += gridDim.x) {
+        const int g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+        const TcGroup& G = p.grp[g];
+        const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
+        const uint32_t idesc = G.idesc;
+        const uint64_t adesc = G.a_mn ? smem_desc(base, TC_MN_CHUNK_BYTES, 1024) : smem_desc(base, 16, 1024);
+        const uint64_t bdesc =
+            G.b_mn ? smem_desc(base + TC_A_BYTES, TC_MN_CHUNK_BYTES, 1024) : smem_desc(base + TC_A_BYTES, 16, 1024);
+        const uint32_t astep = G.a_mn ? (2048u >> 4) : (32u >> 4);  // one K=16 slice, in 16-byte units
+        const uint32_t bstep = G.b_mn ? (2048u >> 4) : (32u >> 4);
+        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * TC_BN;
+        uint32_t accum = 0;
+        for (int kb = 0; kb < nkb; ++kb) {
           if (!mbar_wait(full_bar(stage), phase, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          if (lane == 0) {
-            const uint32_t sa = base + stage * TC_STAGE_BYTES;
-            const uint32_t sb = sa + TC_A_BYTES;
+          const uint32_t so = (uint32_t)(stage * TC_STAGE_BYTES) >> 4;
 #pragma unroll
-            for (int k = 0; k < TC_BK / 16; ++k) {
-              const uint64_t ad = G.a_mn ? smem_desc(sa + k * 2048, TC_MN_CHUNK_BYTES, 1024)
-                                         : smem_desc(sa + k * 32, 16, 1024);
-              const uint64_t bd = G.b_mn ? smem_desc(sb + k * 2048, TC_MN_CHUNK_BYTES, 1024)
-                                         : smem_desc(sb + k * 32, 16, 1024);
-              tc_mma(d_tmem, ad, bd, G.idesc, accum);
-              accum = 1;
-            }
-            tc_commit(empty_bar(stage));
+          for (int k = 0; k < TC_BK / 16; ++k) {
+            tc_mma(d_tmem, adesc + so + k * astep, bdesc + so + k * bstep, idesc, accum);
+            accum = 1;
           }
-          __syncwarp();
+          tc_commit(empty_bar(stage));
           issued_any = true;
           if (++stage == TC_STAGES) { stage = 0; phase ^= 1u; }
         }
+        if (!ok) break;
+        tc_commit(tfull_bar(acc));
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
-      if (!ok) break;
-      if (lane == 0) tc_commit(tfull_bar(acc));
-      __syncwarp();
-      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      if (!ok && issued_any) {
+        // Wait for this thread's MMAs to finish before TMEM is freed.
+        tc_commit(drain_bar);
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < kWaitNs) {}
+      }
     }
-    if (!ok && issued_any) {
-      // Wait for this thread's MMAs to finish before TMEM is freed.
-      if (lane == 0) tc_commit(drain_bar);
-      __syncwarp();
-      const uint64_t t0 = global_timer_ns();
-      while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < kWaitNs) {}
-    }
+    __syncwarp();
   } else {
     // ------------------------------------------------ epilogue (warps 2..9)
     const int q = warp & 3;             // TMEM lane quadrant this warp may access
@@ -486,56 +487,51 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (even CTA only)
-    if (leader) {
+    // ------------------------------------------------ MMA issuer (one thread of the even CTA)
+    if (leader && lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true, issued_any = false;
       for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
-        int g, m0, n0;
-        decode_tile2(p, tile, g, m0, n0);
+        const int g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
         const TcGroup& G = p.grp[g];
+        const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
+        const uint32_t idesc = G.idesc;
+        const uint64_t adesc = G.a_mn ? smem_desc(base, TC_MN_CHUNK_BYTES, 1024) : smem_desc(base, 16, 1024);
+        const uint64_t bdesc =
+            G.b_mn ? smem_desc(base + T2_A_BYTES, TC_MN_CHUNK_BYTES, 1024) : smem_desc(base + T2_A_BYTES, 16, 1024);
+        const uint32_t astep = G.a_mn ? (2048u >> 4) : (32u >> 4);
+        const uint32_t bstep = G.b_mn ? (2048u >> 4) : (32u >> 4);
         if (!mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * TC_BN;
         uint32_t accum = 0;
-        for (int s = 0; s < G.nseg && ok; ++s) {
-          for (int kb = 0; kb < G.kb[s]; ++kb) {
-            if (!mbar_wait_cluster(full_bar(stage), phase, abort_flag)) { ok = false; break; }
-            tc_fence_after();
-            if (lane == 0) {
-              const uint32_t sa = base + stage * T2_STAGE_BYTES;
-              const uint32_t sb = sa + T2_A_BYTES;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!mbar_wait_cluster(full_bar(stage), phase, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t so = (uint32_t)(stage * T2_STAGE_BYTES) >> 4;
 #pragma unroll
-              for (int k = 0; k < TC_BK / 16; ++k) {
-                const uint64_t ad = G.a_mn ? smem_desc(sa + k * 2048, TC_MN_CHUNK_BYTES, 1024)
-                                           : smem_desc(sa + k * 32, 16, 1024);
-                const uint64_t bd = G.b_mn ? smem_desc(sb + k * 2048, TC_MN_CHUNK_BYTES, 1024)
-                                           : smem_desc(sb + k * 32, 16, 1024);
-                tc_mma_pair(d_tmem, ad, bd, G.idesc, accum);
-                accum = 1;
-              }
-              tc_commit_pair_both(empty_bar(stage));
-            }
-            __syncwarp();
-            issued_any = true;
-            if (++stage == T2_STAGES) { stage = 0; phase ^= 1u; }
+          for (int k = 0; k < TC_BK / 16; ++k) {
+            tc_mma_pair(d_tmem, adesc + so + k * astep, bdesc + so + k * bstep, idesc, accum);
+            accum = 1;
           }
+          tc_commit_pair_both(empty_bar(stage));
+          issued_any = true;
+          if (++stage == T2_STAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        if (lane == 0) tc_commit_pair_both(tfull_bar(acc));
-        __syncwarp();
+        tc_commit_pair_both(tfull_bar(acc));
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
       if (!ok && issued_any) {
-        if (lane == 0) tc_commit_pair_local(drain_bar);
-        __syncwarp();
+        tc_commit_pair_local(drain_bar);
         const uint64_t t0 = global_timer_ns();
         while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < kWaitNs) {}
       }
     }
+    __syncwarp();
   } else {
     // ------------------------------------------------ epilogue (warps 2..9, both CTAs)
     const int q = warp & 3;
