@@ -24,10 +24,10 @@ def _dev_bf16(a, ld_mult=8):
 
 
 SHAPES = [(128, 256, 64), (256, 512, 1024), (300, 520, 200), (1, 17, 8), (129, 257, 65), (640, 1000, 768),
-          (2048, 2304, 512)]  # the last spans more 256x256 tiles than there are CTA pairs on the GPU
+          (2048, 2304, 512), (4000, 2304, 256)]  # the last two span more 256x256 tiles than there are CTA pairs
 
 
-@pytest.mark.parametrize("engine", ["tcgen05", "tcgen05_pair"])
+@pytest.mark.parametrize("engine", ["tcgen05", "tcgen05_pair", "tcgen05_mc"])
 @pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (0, 1), (1, 0), (1, 1)])
 @pytest.mark.parametrize("M,N,K", SHAPES)
 def test_gemm_tcgen05_matches_matmul(M, N, K, a_mn, b_mn, engine):
