@@ -81,6 +81,18 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
+// One AdamW update (Loshchilov & Hutter, decoupled weight decay w) of a
+// parameter p with gradient g and moments m, v; rbc1 = 1 / (1 - beta1^t),
+// rbc2 = 1 / (1 - beta2^t).  Shared by the optimizer kernel and the fused
+// weight-gradient GEMM epilogue so both give identical results.
+__device__ __forceinline__ void adamw_elem(float& p, float& m, float& v, float g, float lr, float b1, float b2,
+                                           float eps, float w, float rbc1, float rbc2) {
+  m = b1 * m + (1.f - b1) * g;
+  v = b2 * v + (1.f - b2) * g * g;
+  const float mh = m * rbc1, vh = v * rbc2;
+  p -= lr * (mh / (sqrtf(vh) + eps) + w * p);
+}
+
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));

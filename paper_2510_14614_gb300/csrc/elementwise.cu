@@ -292,13 +292,8 @@ __global__ void adamw_kernel(size_t n, size_t n_decay, float* __restrict__ p, co
     float4 pp = load4(p + e), gg = load4(g + e), mm = load4(m + e), vv = load4(v + e);
     float* pa = &pp.x; float* ga = &gg.x; float* ma = &mm.x; float* va = &vv.x;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      ma[j] = b1 * ma[j] + (1.f - b1) * ga[j];
-      va[j] = b2 * va[j] + (1.f - b2) * ga[j] * ga[j];
-      const float mh = ma[j] * rbc1, vh = va[j] * rbc2;
-      const float w = (e + j < n_decay) ? wd : 0.f;
-      pa[j] -= lr * (mh / (sqrtf(vh) + eps) + w * pa[j]);
-    }
+    for (int j = 0; j < 4; ++j)
+      adamw_elem(pa[j], ma[j], va[j], ga[j], lr, b1, b2, eps, (e + j < n_decay) ? wd : 0.f, rbc1, rbc2);
     store4(p + e, pp); store4(m + e, mm); store4(v + e, vv);
     if (shadow) store4(shadow + e, pp);
   }

@@ -15,15 +15,42 @@ template <> __device__ __forceinline__ float epi_gelu_grad<bf16>(float x) { retu
 
 // ---- compile-time specialised epilogue arithmetic
 // Which inputs an epilogue reads, as bits of a compile-time KIND.
+// EK_ADAMW (a weight gradient with the optimizer update fused) reads nothing
+// else and is never part of EK_ANY.
 enum EpiKind {
   EK_BIAS = 1, EK_BIAS2 = 2, EK_DGELU = 4, EK_PRE = 8, EK_RESID = 16, EK_RESID2 = 32, EK_GELU = 64,
-  EK_ANY = 127  // every input present-or-null, tested at run time
+  EK_ANY = 127,  // every input present-or-null, tested at run time
+  EK_ADAMW = 128
 };
 
 __host__ __device__ inline int epi_kind(const EpiParams& e) {
+  if (e.op == EPI_ADAMW) return EK_ADAMW;
   return (e.bias ? EK_BIAS : 0) | (e.bias2 ? EK_BIAS2 : 0) | (e.op == EPI_DGELU ? EK_DGELU : 0) |
          (e.pre_f32 ? EK_PRE : 0) | (e.resid ? EK_RESID : 0) | (e.resid2 ? EK_RESID2 : 0) |
          (e.op == EPI_GELU ? EK_GELU : 0);
+}
+
+// AdamW applied to the parameter elements (row, c..c+n) of an EPI_ADAMW
+// epilogue, given their gradient g (the value just stored to `out`).
+template <int NE>
+__device__ __forceinline__ void epi_adamw(const EpiParams& e, int row, int c, const float* g) {
+  const long o = (long)row * e.ldo + c;
+  if (NE == 4) {
+    float4 p = load4(e.opt_p + o), m = load4(e.opt_m + o), v = load4(e.opt_v + o);
+    adamw_elem(p.x, m.x, v.x, g[0], e.opt_lr, e.opt_b1, e.opt_b2, e.opt_eps, e.opt_wd, e.opt_rbc1, e.opt_rbc2);
+    adamw_elem(p.y, m.y, v.y, g[1], e.opt_lr, e.opt_b1, e.opt_b2, e.opt_eps, e.opt_wd, e.opt_rbc1, e.opt_rbc2);
+    adamw_elem(p.z, m.z, v.z, g[2], e.opt_lr, e.opt_b1, e.opt_b2, e.opt_eps, e.opt_wd, e.opt_rbc1, e.opt_rbc2);
+    adamw_elem(p.w, m.w, v.w, g[3], e.opt_lr, e.opt_b1, e.opt_b2, e.opt_eps, e.opt_wd, e.opt_rbc1, e.opt_rbc2);
+    store4(e.opt_p + o, p); store4(e.opt_m + o, m); store4(e.opt_v + o, v);
+    if (e.opt_sh) store4(reinterpret_cast<bf16*>(e.opt_sh) + o, p);
+  } else {
+    for (int j = 0; j < NE; ++j) {
+      float p = e.opt_p[o + j], m = e.opt_m[o + j], v = e.opt_v[o + j];
+      adamw_elem(p, m, v, g[j], e.opt_lr, e.opt_b1, e.opt_b2, e.opt_eps, e.opt_wd, e.opt_rbc1, e.opt_rbc2);
+      e.opt_p[o + j] = p; e.opt_m[o + j] = m; e.opt_v[o + j] = v;
+      if (e.opt_sh) reinterpret_cast<bf16*>(e.opt_sh)[o + j] = __float2bfloat16_rn(p);
+    }
+  }
 }
 
 // The pointers and strides an epilogue reads, held by value so that they stay
@@ -155,6 +182,7 @@ __device__ __forceinline__ void epi_row(const EpiParams& e, int M, int N, int ro
         float* p = reinterpret_cast<float*>(e.out) + (long)row * e.ldo + c;
         if (e.out_mode == OUT_F32_ACCUM) { float4 q = load4(p); o.x += q.x; o.y += q.y; o.z += q.z; o.w += q.w; }
         store4(p, o);
+        if (e.op == EPI_ADAMW) epi_adamw<4>(e, row, c, &o.x);
       }
     } else {
       for (int j = 0; j < 4 && c + j < N; ++j) {
@@ -174,6 +202,7 @@ __device__ __forceinline__ void epi_row(const EpiParams& e, int M, int N, int ro
         } else {
           float* p = reinterpret_cast<float*>(e.out) + (long)row * e.ldo + cc;
           *p = (e.out_mode == OUT_F32_ACCUM) ? *p + y : y;
+          if (e.op == EPI_ADAMW) epi_adamw<1>(e, row, cc, &y);
         }
       }
     }

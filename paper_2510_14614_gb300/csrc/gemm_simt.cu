@@ -11,7 +11,7 @@ constexpr int SB_M = 64, SB_N = 64, SB_K = 16;
 
 struct SimtParams {
   GemmCall c;
-  int tiles[2];  // tiles per group
+  int tiles[kMaxGemmGroups];  // tiles per group
 };
 
 template <typename in_t>
@@ -27,7 +27,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __grid_constant__ 
   __shared__ float Bs[SB_K][SB_N + 4];
   int tile = blockIdx.x;
   int g = 0;
-  if (tile >= p.tiles[0]) { tile -= p.tiles[0]; g = 1; }
+  while (g + 1 < kMaxGemmGroups && tile >= p.tiles[g]) { tile -= p.tiles[g]; ++g; }
   const GemmGroupDesc& G = p.c.g[g];
   const int mt = (G.M + SB_M - 1) / SB_M;
   const int m0 = (tile % mt) * SB_M, n0 = (tile / mt) * SB_N;
@@ -67,7 +67,8 @@ int gemm_simt(const GemmCall& c, int in_bf16, int act_bf16, cudaStream_t s, std:
   SimtParams p;
   p.c = c;
   int total = 0;
-  for (int g = 0; g < 2; ++g) {
+  if (c.ngroups < 1 || c.ngroups > kMaxGemmGroups) { if (msg) *msg = "GEMM launch needs 1 to 4 groups"; return 1; }
+  for (int g = 0; g < kMaxGemmGroups; ++g) {
     p.tiles[g] = 0;
     if (g < c.ngroups) {
       const GemmGroupDesc& G = c.g[g];

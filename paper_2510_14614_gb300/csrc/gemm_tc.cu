@@ -61,9 +61,10 @@ struct TcGroup {
   EpiParams epi;
 };
 
+constexpr int kMaxMaps = 20;  // operand maps (2 per K segment) and output maps (up to 2) of all groups
 struct TcParams {
-  CUtensorMap maps[12];
-  TcGroup grp[2];
+  CUtensorMap maps[kMaxMaps];
+  TcGroup grp[kMaxGemmGroups];
   int ngroups, total_tiles;
   int* err;
 };
@@ -83,10 +84,101 @@ struct EpiOut {
   int M, N, out_tma, out_f32, out_accum, omap, omap2, gelu;
 };
 
+// EPI_ADAMW chunk: the gradient tile is transposed through the warp's buffer so
+// that each row segment is read and written with coalesced 16-byte accesses:
+// gradient store, then the AdamW update of the weight (master, moments, bf16
+// copy).  The optimizer's operands are read from the parameter block once per
+// chunk.
+__device__ __forceinline__ void epi_adamw_chunk(const EpiParams* ep, int M, int N, float4* stage, int lane, int row0,
+                                                int col0, const uint32_t* r) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    stage[lane * 8 + (j ^ (lane & 7))] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                                     __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+  __syncwarp();
+  float* const g = reinterpret_cast<float*>(ep->out);
+  float* const pp = ep->opt_p;
+  float* const mm = ep->opt_m;
+  float* const vv = ep->opt_v;
+  bf16* const sh = reinterpret_cast<bf16*>(ep->opt_sh);
+  const long ld = ep->ldo;
+  const float lr = ep->opt_lr, b1 = ep->opt_b1, b2 = ep->opt_b2, eps = ep->opt_eps, wd = ep->opt_wd;
+  const float rbc1 = ep->opt_rbc1, rbc2 = ep->opt_rbc2;
+  const int rb = lane >> 3, ch = lane & 7;
+  if (row0 + 32 <= M && col0 + 32 <= N) {
+    // Interior chunk: every lane first asks L2 for its row's 128-byte segments
+    // of the three optimizer arrays (the whole 32x32 chunk is then in flight
+    // at once, at no register cost), then two row groups at a time are loaded,
+    // updated and stored.
+    {
+      const long o = (long)(row0 + lane) * ld + col0;
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(pp + o));
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(mm + o));
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(vv + o));
+    }
+#pragma unroll 1
+    for (int h0 = 0; h0 < 8; h0 += 2) {
+      float4 P[2], Mv[2], Vv[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const long o = (long)(row0 + (h0 + j) * 4 + rb) * ld + col0 + ch * 4;
+        P[j] = load4(pp + o); Mv[j] = load4(mm + o); Vv[j] = load4(vv + o);
+      }
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int rr = (h0 + j) * 4 + rb;
+        const long o = (long)(row0 + rr) * ld + col0 + ch * 4;
+        const float4 v4 = stage[rr * 8 + (ch ^ (rr & 7))];
+        store4(g + o, v4);
+        adamw_elem(P[j].x, Mv[j].x, Vv[j].x, v4.x, lr, b1, b2, eps, wd, rbc1, rbc2);
+        adamw_elem(P[j].y, Mv[j].y, Vv[j].y, v4.y, lr, b1, b2, eps, wd, rbc1, rbc2);
+        adamw_elem(P[j].z, Mv[j].z, Vv[j].z, v4.z, lr, b1, b2, eps, wd, rbc1, rbc2);
+        adamw_elem(P[j].w, Mv[j].w, Vv[j].w, v4.w, lr, b1, b2, eps, wd, rbc1, rbc2);
+        store4(pp + o, P[j]); store4(mm + o, Mv[j]); store4(vv + o, Vv[j]);
+        if (sh) store4(sh + o, P[j]);
+      }
+    }
+    __syncwarp();
+    return;
+  }
+#pragma unroll 1
+  for (int it = 0; it < 8; ++it) {
+    const int rr = it * 4 + rb;
+    const int row = row0 + rr, c = col0 + ch * 4;
+    if (row >= M || c >= N) continue;
+    const float4 v4 = stage[rr * 8 + (ch ^ (rr & 7))];
+    const long o = (long)row * ld + c;
+    if (c + 4 <= N) {
+      store4(g + o, v4);
+      float4 p = load4(pp + o), m = load4(mm + o), v = load4(vv + o);
+      adamw_elem(p.x, m.x, v.x, v4.x, lr, b1, b2, eps, wd, rbc1, rbc2);
+      adamw_elem(p.y, m.y, v.y, v4.y, lr, b1, b2, eps, wd, rbc1, rbc2);
+      adamw_elem(p.z, m.z, v.z, v4.z, lr, b1, b2, eps, wd, rbc1, rbc2);
+      adamw_elem(p.w, m.w, v.w, v4.w, lr, b1, b2, eps, wd, rbc1, rbc2);
+      store4(pp + o, p); store4(mm + o, m); store4(vv + o, v);
+      if (sh) store4(sh + o, p);
+    } else {
+      const float gv[4] = {v4.x, v4.y, v4.z, v4.w};
+      for (int j = 0; j < 4 && c + j < N; ++j) {
+        g[o + j] = gv[j];
+        float p = pp[o + j], m = mm[o + j], v = vv[o + j];
+        adamw_elem(p, m, v, gv[j], lr, b1, b2, eps, wd, rbc1, rbc2);
+        pp[o + j] = p; mm[o + j] = m; vv[o + j] = v;
+        if (sh) sh[o + j] = __float2bfloat16_rn(p);
+      }
+    }
+  }
+  __syncwarp();
+}
+
 template <typename act_t, int KIND>
 __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep, const EpiIn q, const EpiOut o,
                                           float4* stage, uint32_t stage_s, int lane, int row0, int col0,
                                           const uint32_t* r) {
+  if constexpr (KIND == EK_ADAMW) {
+    epi_adamw_chunk(ep, o.M, o.N, stage, lane, row0, col0, r);
+    return;
+  }
   if (!o.out_tma) {
 #pragma unroll
     for (int j = 0; j < 8; ++j)
@@ -168,6 +260,7 @@ __device__ __forceinline__ void epi_chunk_dispatch(int kind, const TcParams& p, 
     case EK_BIAS | EK_RESID: epi_chunk<act_t, EK_BIAS | EK_RESID>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
     case EK_BIAS | EK_BIAS2 | EK_RESID:
       epi_chunk<act_t, EK_BIAS | EK_BIAS2 | EK_RESID>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_ADAMW: epi_chunk<act_t, EK_ADAMW>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
     default: epi_chunk<act_t, EK_ANY>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
   }
 }
@@ -179,11 +272,20 @@ __device__ __forceinline__ EpiOut epi_out_of(const TcGroup& G) {
   return o;
 }
 
+// Group of a tile index: groups own consecutive tile ranges in group order.
+__device__ __forceinline__ int group_of(const TcParams& p, int tile) {
+  int g = 0;
+#pragma unroll
+  for (int k = 1; k < kMaxGemmGroups; ++k)
+    if (k < p.ngroups && tile >= p.grp[k].tile_start) g = k;
+  return g;
+}
+
 // MC: a cluster of two CTAs owns a 256-row band of output tiles; CTA `rank`
 // computes rows m0 + 128 * rank.
 template <bool MC>
 __device__ __forceinline__ void decode_tile(const TcParams& p, int tile, uint32_t rank, int& g, int& m0, int& n0) {
-  g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+  g = group_of(p, tile);
   const TcGroup& G = p.grp[g];
   const int local = tile - G.tile_start;
   m0 = (local % G.m_tiles) * (MC ? 2 * TC_BM : TC_BM) + (int)rank * TC_BM;
@@ -321,7 +423,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       uint32_t acc_phase = 0;
       bool ok = true, issued_any = false;
       for (int tile = unit; tile < p.total_tiles && ok; tile += nunits) {
-        const int g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+        const int g = group_of(p, tile);
         const TcGroup& G = p.grp[g];
         const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
         const uint32_t idesc = G.idesc;
@@ -421,7 +523,7 @@ constexpr int T2_SMEM = T2_STAGES * T2_STAGE_BYTES + TC_EPI_WARPS * TC_EPI_STAGE
 constexpr int T2_TILE = 256;
 
 __device__ __forceinline__ void decode_tile2(const TcParams& p, int tile, int& g, int& m0, int& n0) {
-  g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+  g = group_of(p, tile);
   const TcGroup& G = p.grp[g];
   const int local = tile - G.tile_start;
   m0 = (local % G.m_tiles) * T2_TILE;
@@ -531,7 +633,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       uint32_t acc_phase = 0;
       bool ok = true, issued_any = false;
       for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
-        const int g = (p.ngroups > 1 && tile >= p.grp[1].tile_start) ? 1 : 0;
+        const int g = group_of(p, tile);
         const TcGroup& G = p.grp[g];
         const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
         const uint32_t idesc = G.idesc;
@@ -783,6 +885,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
   TcParams p;
   memset(&p, 0, sizeof(p));
   int nmaps = 0, tiles = 0;
+  if (c.ngroups < 1 || c.ngroups > kMaxGemmGroups) { if (msg) *msg = "GEMM launch needs 1 to 4 groups"; return 1; }
   p.ngroups = c.ngroups;
   for (int g = 0; g < c.ngroups; ++g) {
     const GemmGroupDesc& G = c.g[g];
@@ -808,6 +911,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
         return 1;
       }
       T.kb[sg] = (S.K + TC_BK - 1) / TC_BK;
+      if (nmaps + 2 > kMaxMaps) { if (msg) *msg = "too many GEMM operands in one launch"; return 1; }
       // A: logical [M, K]
       if (S.A.mn_major) {
         if (!encode_map(&p.maps[nmaps], S.A.ptr, G.M, S.K, S.A.ld, 64, TC_BK, msg)) return 1;
@@ -827,14 +931,21 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     {
       const int k = epi_kind(e);
       const bool special = k == 0 || k == EK_BIAS || k == (EK_BIAS | EK_GELU) || k == EK_DGELU ||
-                           k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID);
+                           k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID) || k == EK_ADAMW;
       T.kind = special ? k : EK_ANY;
+    }
+    if (e.op == EPI_ADAMW &&
+        (e.out_mode != OUT_F32 || !e.opt_p || !e.opt_m || !e.opt_v || !check_ld(e.ldo, e.opt_p) ||
+         !check_ld(e.ldo, e.opt_m) || !check_ld(e.ldo, e.opt_v) ||
+         (e.opt_sh && (reinterpret_cast<uintptr_t>(e.opt_sh) & 7)))) {
+      if (msg) *msg = "fused AdamW epilogue needs an fp32 gradient output and aligned optimizer arrays";
+      return 1;
     }
     T.out_f32 = e.out_mode != OUT_ACT && e.op != EPI_GELU;
     T.out_accum = e.out_mode == OUT_F32_ACCUM;
     T.out_tma = 0;
     T.omap = T.omap2 = 0;
-    if (nmaps + 2 <= 12 && encode_out_map(&p.maps[nmaps], e.out, T.out_f32, G.N, G.M, e.ldo)) {
+    if (e.op != EPI_ADAMW && nmaps + 2 <= kMaxMaps && encode_out_map(&p.maps[nmaps], e.out, T.out_f32, G.N, G.M, e.ldo)) {
       T.omap = nmaps;
       bool ok = true;
       if (e.op == EPI_GELU) {

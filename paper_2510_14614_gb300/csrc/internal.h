@@ -16,8 +16,11 @@ enum DevErr { DEV_OK = 0, DEV_ERR_TOKEN = 1, DEV_ERR_TIMEOUT = 2 };
 // A[k*ld + m] (MN-major); B operand element (n,k) at B[n*ld + k] (K-major) or
 // B[k*ld + n] (MN-major).  A group may chain two K segments (two operand pairs
 // summed into one accumulator: the fused [ctx | g] x [W_o ; W_down] residual
-// GEMM), and one launch may run two independent groups.
-enum EpiOp { EPI_NONE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
+// GEMM), and one launch may run up to four independent groups (tiles in group
+// order).
+// EPI_ADAMW: the GEMM computes the gradient of a weight matrix (stored to `out`,
+// fp32, OUT_F32) and the epilogue also applies AdamW to that weight in place.
+enum EpiOp { EPI_NONE = 0, EPI_GELU = 1, EPI_DGELU = 2, EPI_ADAMW = 3 };
 enum OutMode { OUT_ACT = 0, OUT_F32 = 1, OUT_F32_ACCUM = 2 };
 
 struct EpiParams {
@@ -30,12 +33,18 @@ struct EpiParams {
   const float* resid; long ldr;             // fp32 [M, N] added after pre_f32
   const float* resid2; long ldr2;
   const void* aux; long ldx;                // DGELU: pre-activation h (activation type)
+  // ADAMW: fp32 master weights, moments and the bf16 copy the GEMMs read (or
+  // null), all [M, N] with row pitch ldo; decoupled weight decay wd; rbc1 and
+  // rbc2 are 1 / (1 - beta^t).
+  float* opt_p; float* opt_m; float* opt_v; void* opt_sh;
+  float opt_lr, opt_b1, opt_b2, opt_eps, opt_wd, opt_rbc1, opt_rbc2;
 };
 
 struct GemmOperand { const void* ptr; long ld; int mn_major; };
 struct GemmSeg { GemmOperand A, B; int K; };
 struct GemmGroupDesc { int M, N; int nseg; GemmSeg seg[2]; EpiParams epi; };
-struct GemmCall { int ngroups; GemmGroupDesc g[2]; };
+constexpr int kMaxGemmGroups = 4;
+struct GemmCall { int ngroups; GemmGroupDesc g[kMaxGemmGroups]; };
 
 // Plain fp32-FMA tiled GEMM (debug precision; also a GPU cross-check).
 // in_bf16: operands are bf16 (else fp32); act_bf16: activation outputs bf16.

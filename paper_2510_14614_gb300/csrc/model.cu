@@ -17,6 +17,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <initializer_list>
 #include <vector>
 
 #include "../../include/fal.h"
@@ -70,6 +71,10 @@ struct fal_handle {
   int state = 0;  // 0 fresh, 1 after forward, 2 after backward
   bool has_loss = false;
   long step_t = 0;
+  // fal_train_step: the weight-gradient GEMMs of the block matrices also apply
+  // AdamW (bias corrections of step step_t).
+  bool fuse_opt = false;
+  float opt_rbc1 = 1.f, opt_rbc2 = 1.f;
 
   std::vector<fal_tensor_info> tensors;
   size_t n_params = 0, n_decay = 0;
@@ -78,7 +83,13 @@ struct fal_handle {
 
   // workspace views
   float *P = nullptr, *G = nullptr, *Mo = nullptr, *Vo = nullptr;
-  void* Sh = nullptr;
+  // bf16 copies of the parameters read by the GEMMs (bf16 path), two buffers:
+  // the forward and backward read Shb[sh_cur]; AdamW writes the updated copy
+  // into the other one, which becomes current after the step.  With the
+  // optimizer fused into the weight-gradient GEMMs, a data-gradient GEMM that
+  // runs in the same launch still reads this step's weights.
+  void* Shb[2] = {nullptr, nullptr};
+  int sh_cur = 0;
   int32_t *tok = nullptr, *tgt = nullptr;
   int* dev_err = nullptr;
   float *loss = nullptr, *loss_rows = nullptr;
@@ -247,7 +258,8 @@ void carve(fal_handle* h, uint8_t* base) {
   h->G = b.take<float>(h->n_params);
   h->Mo = b.take<float>(h->n_params);
   h->Vo = b.take<float>(h->n_params);
-  h->Sh = h->bf ? b.take<uint8_t>(h->n_params * 2) : nullptr;
+  h->Shb[0] = h->bf ? b.take<uint8_t>(h->n_params * 2) : nullptr;
+  h->Shb[1] = h->bf ? b.take<uint8_t>(h->n_params * 2) : nullptr;
   h->tok = b.take<int32_t>(BT);
   h->tgt = b.take<int32_t>(BT);
   h->dev_err = b.take<int>(4);
@@ -337,11 +349,38 @@ GemmCall call1(int M, int N, GemmSeg s0, const EpiParams& e) {
   return c;
 }
 
+// One launch running the groups of several calls (independent contractions),
+// tiles in argument order.  Weight-gradient groups go first: their epilogues
+// (fp32 stores, fused AdamW) then overlap the data-gradient main loops, and
+// the wave tails of the separate launches disappear.
+GemmCall group_calls(std::initializer_list<GemmCall> calls) {
+  GemmCall out;
+  memset(&out, 0, sizeof(out));
+  for (const GemmCall& c : calls)
+    for (int g = 0; g < c.ngroups && out.ngroups < kMaxGemmGroups; ++g) out.g[out.ngroups++] = c.g[g];
+  return out;
+}
+
 float* Pp(fal_handle* h, size_t off) { return off == NPOS ? nullptr : h->P + off; }
 float* Gp(fal_handle* h, size_t off) { return off == NPOS ? nullptr : h->G + off; }
 // GEMM weight operand: bf16 copy on the bf16 path, fp32 master on the debug path.
 const void* Wp(fal_handle* h, size_t off) {
-  return h->bf ? (const void*)((const uint8_t*)h->Sh + off * 2) : (const void*)(h->P + off);
+  return h->bf ? (const void*)((const uint8_t*)h->Shb[h->sh_cur] + off * 2) : (const void*)(h->P + off);
+}
+
+// Epilogue of the weight-gradient GEMM of the matrix at offset w ([rows, ld]):
+// the fp32 gradient, and under fal_train_step the AdamW update of the matrix.
+EpiParams wgrad_out(fal_handle* h, size_t w, long ld) {
+  EpiParams e = epi_out(Gp(h, w), ld, OUT_F32);
+  if (h->fuse_opt) {
+    const fal_config& c = h->cfg;
+    e.op = EPI_ADAMW;
+    e.opt_p = h->P + w; e.opt_m = h->Mo + w; e.opt_v = h->Vo + w;
+    e.opt_sh = h->bf ? (void*)((uint8_t*)h->Shb[h->sh_cur ^ 1] + w * 2) : nullptr;
+    e.opt_lr = c.lr; e.opt_b1 = c.beta1; e.opt_b2 = c.beta2; e.opt_eps = c.eps; e.opt_wd = c.weight_decay;
+    e.opt_rbc1 = h->opt_rbc1; e.opt_rbc2 = h->opt_rbc2;
+  }
+  return e;
 }
 
 cudaEvent_t pool_event(fal_handle* h) {
@@ -571,11 +610,13 @@ void mlp_backward(Ctx& c, int i, const float* dXn, const void* dXn_act, cudaStre
   const int BT = (int)h->BT, d = h->d, F = h->F;
   EpiParams e = epi_out(h->dh, F, OUT_ACT);
   e.op = EPI_DGELU; e.aux = A.h; e.ldx = F;
-  gemm(c, call1(BT, F, dgrad_seg(h, dXn_act, d, p.w_down, F), e), s, "MLP down dgrad");
-  gemm(c, call1(d, F, wgrad_seg(h, dXn_act, d, A.g, F), epi_out(Gp(h, p.w_down), F, OUT_F32)), s, "MLP down wgrad");
+  gemm(c, group_calls({call1(d, F, wgrad_seg(h, dXn_act, d, A.g, F), wgrad_out(h, p.w_down, F)),
+                       call1(BT, F, dgrad_seg(h, dXn_act, d, p.w_down, F), e)}),
+       s, "MLP down wgrad + dgrad");
   colsum_(c, s, part, dXn, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_down), nullptr, 0);
-  gemm(c, call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32)), s, "MLP up dgrad");
-  gemm(c, call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), epi_out(Gp(h, p.w_up), d, OUT_F32)), s, "MLP up wgrad");
+  gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), wgrad_out(h, p.w_up, d)),
+                       call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
+       s, "MLP up wgrad + dgrad");
   colsum_(c, s, part, h->dh, 1, F, F, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_up), nullptr, 0);
 }
 
@@ -586,8 +627,9 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   const LayerP& p = h->lp[i];
   const int BT = (int)h->BT, d = h->d;
   if (!skip_wo) {
-    gemm(c, call1(BT, d, dgrad_seg(h, da_act, d, p.w_o, d), epi_out(h->dctx, d, OUT_ACT)), s, "attention out dgrad");
-    gemm(c, call1(d, d, wgrad_seg(h, da_act, d, A.ctx, d), epi_out(Gp(h, p.w_o), d, OUT_F32)), s, "attention out wgrad");
+    gemm(c, group_calls({call1(d, d, wgrad_seg(h, da_act, d, A.ctx, d), wgrad_out(h, p.w_o, d)),
+                         call1(BT, d, dgrad_seg(h, da_act, d, p.w_o, d), epi_out(h->dctx, d, OUT_ACT))}),
+         s, "attention out wgrad + dgrad");
     colsum_(c, s, part, da, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o), nullptr, 0);
   }
   if (!c.ok()) return;
@@ -596,8 +638,9 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dq_acc, h->dvec,
                    h->dev_err, s, &h->err),
           "attention backward");
-  gemm(c, call1(BT, d, dgrad_seg(h, h->dqkv, 3 * d, p.w_qkv, d), epi_out(h->dU, d, OUT_F32)), s, "QKV dgrad");
-  gemm(c, call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), epi_out(Gp(h, p.w_qkv), d, OUT_F32)), s, "QKV wgrad");
+  gemm(c, group_calls({call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), wgrad_out(h, p.w_qkv, d)),
+                       call1(BT, d, dgrad_seg(h, h->dqkv, 3 * d, p.w_qkv, d), epi_out(h->dU, d, OUT_F32))}),
+       s, "QKV wgrad + dgrad");
   colsum_(c, s, part, h->dqkv, 1, 3L * d, 3 * d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_qkv),
           nullptr, 0);
 }
@@ -619,33 +662,24 @@ void layer_backward(Ctx& c, int i) {
   cudaStream_t s = h->sm;
   // dX / dX_act hold the gradient w.r.t. X_{i+1} on entry and X_i on exit.
   if (var == FAL_FAL && i >= 1) {
-    // One grouped dgrad launch: [dctx | dh] = dX [W_o | W_down] (dh with gelu'),
-    // one grouped wgrad launch: [dW_o | dW_down] = dX^T [ctx | g].
-    GemmCall dg;
-    memset(&dg, 0, sizeof(dg));
-    dg.ngroups = 2;
-    dg.g[0].M = BT; dg.g[0].N = d; dg.g[0].nseg = 1; dg.g[0].seg[0] = dgrad_seg(h, h->dX_act, d, p.w_o, d);
-    dg.g[0].epi = epi_out(h->dctx, d, OUT_ACT);
-    dg.g[1].M = BT; dg.g[1].N = F; dg.g[1].nseg = 1; dg.g[1].seg[0] = dgrad_seg(h, h->dX_act, d, p.w_down, F);
-    dg.g[1].epi = epi_out(h->dh, F, OUT_ACT);
-    dg.g[1].epi.op = EPI_DGELU; dg.g[1].epi.aux = A.h; dg.g[1].epi.ldx = F;
-    gemm(c, dg, s, "fused residual dgrad");
-    GemmCall wg;
-    memset(&wg, 0, sizeof(wg));
-    wg.ngroups = 2;
-    wg.g[0].M = d; wg.g[0].N = d; wg.g[0].nseg = 1; wg.g[0].seg[0] = wgrad_seg(h, h->dX_act, d, A.ctx, d);
-    wg.g[0].epi = epi_out(Gp(h, p.w_o), d, OUT_F32);
-    wg.g[1].M = d; wg.g[1].N = F; wg.g[1].nseg = 1; wg.g[1].seg[0] = wgrad_seg(h, h->dX_act, d, A.g, F);
-    wg.g[1].epi = epi_out(Gp(h, p.w_down), F, OUT_F32);
-    gemm(c, wg, s, "fused residual wgrad");
+    // One launch for the fused residual GEMM's gradients:
+    // [dW_o | dW_down] = dX^T [ctx | g] and [dctx | dh] = dX [W_o | W_down] (dh with gelu').
+    EpiParams edh = epi_out(h->dh, F, OUT_ACT);
+    edh.op = EPI_DGELU; edh.aux = A.h; edh.ldx = F;
+    gemm(c, group_calls({call1(d, d, wgrad_seg(h, h->dX_act, d, A.ctx, d), wgrad_out(h, p.w_o, d)),
+                         call1(d, F, wgrad_seg(h, h->dX_act, d, A.g, F), wgrad_out(h, p.w_down, F)),
+                         call1(BT, d, dgrad_seg(h, h->dX_act, d, p.w_o, d), epi_out(h->dctx, d, OUT_ACT)),
+                         call1(BT, F, dgrad_seg(h, h->dX_act, d, p.w_down, F), edh)}),
+         s, "fused residual wgrad + dgrad");
     colsum_(c, s, h->part0, h->dX, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o),
             Gp(h, p.b_down), 0);
     const bool two = h->cfg.schedule == FAL_SCHED_TWO_STREAM && h->ss != h->sm;
     cudaStream_t sa = two ? h->ss : s;
     if (two) fork(h);
     attn_backward(c, i, nullptr, nullptr, sa, two ? h->part1 : h->part0, true);
-    gemm(c, call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32)), s, "MLP up dgrad");
-    gemm(c, call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), epi_out(Gp(h, p.w_up), d, OUT_F32)), s, "MLP up wgrad");
+    gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), wgrad_out(h, p.w_up, d)),
+                         call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
+         s, "MLP up wgrad + dgrad");
     colsum_(c, s, h->part0, h->dh, 1, F, F, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_up),
             nullptr, 0);
     first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
@@ -770,7 +804,8 @@ int fal_create(const fal_config* cfg, void* workspace, size_t bytes, void* strea
   cudaMemsetAsync(h->G, 0, h->n_params * 4, s);
   cudaMemsetAsync(h->Mo, 0, h->n_params * 4, s);
   cudaMemsetAsync(h->Vo, 0, h->n_params * 4, s);
-  if (h->Sh) cudaMemsetAsync(h->Sh, 0, h->n_params * 2, s);
+  for (void* b : h->Shb)
+    if (b) cudaMemsetAsync(b, 0, h->n_params * 2, s);
   cudaMemsetAsync(h->dev_err, 0, 16, s);
   if (cudaStreamSynchronize(s) != cudaSuccess) {
     cudaEventDestroy(h->ev_fork);
@@ -830,16 +865,25 @@ int fal_backward(fal_handle* h) {
   return FAL_OK;
 }
 
+namespace {
+// AdamW over the flat range [begin, end) of the parameter buffer; elements
+// below decay_end get weight decay.
+int adamw_range(fal_handle* h, size_t begin, size_t end, size_t decay_end) {
+  const fal_config& c = h->cfg;
+  const float bc1 = 1.f - (float)pow((double)c.beta1, (double)h->step_t);
+  const float bc2 = 1.f - (float)pow((double)c.beta2, (double)h->step_t);
+  void* sh = h->bf ? (void*)((uint8_t*)h->Shb[h->sh_cur ^ 1] + begin * 2) : nullptr;
+  return adamw(end - begin, decay_end > begin ? decay_end - begin : 0, h->P + begin, h->G + begin, h->Mo + begin,
+               h->Vo + begin, sh, c.lr, c.beta1, c.beta2, c.eps, c.weight_decay, bc1, bc2, h->sm);
+}
+}  // namespace
+
 int fal_step(fal_handle* h) {
   if (!h) return FAL_ERR_ARG;
   if (h->state < 2) return fail(h, FAL_ERR_STATE, "fal_step needs a preceding fal_backward");
   h->step_t += 1;
-  const fal_config& c = h->cfg;
-  const float bc1 = 1.f - (float)pow((double)c.beta1, (double)h->step_t);
-  const float bc2 = 1.f - (float)pow((double)c.beta2, (double)h->step_t);
-  int r = adamw(h->n_params, h->n_decay, h->P, h->G, h->Mo, h->Vo, h->Sh, c.lr, c.beta1, c.beta2, c.eps, c.weight_decay,
-                bc1, bc2, h->sm);
-  if (r) return fail(h, FAL_ERR_CUDA, "AdamW launch failed");
+  if (adamw_range(h, 0, h->n_params, h->n_decay)) return fail(h, FAL_ERR_CUDA, "AdamW launch failed");
+  h->sh_cur ^= 1;
   h->state = 0;
   return FAL_OK;
 }
@@ -847,10 +891,29 @@ int fal_step(fal_handle* h) {
 int fal_train_step(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host) {
   int r = fal_forward(h, tokens, targets, nullptr);
   if (r) return r;
-  r = fal_backward(h);
+  // The block matrices (one contiguous range of the flat buffer, after wte and
+  // wpe) are updated by their weight-gradient GEMMs during the backward; one
+  // AdamW launch per remaining range follows.
+  h->step_t += 1;
+  {
+    const fal_config& c = h->cfg;
+    h->opt_rbc1 = 1.f / (1.f - (float)pow((double)c.beta1, (double)h->step_t));
+    h->opt_rbc2 = 1.f / (1.f - (float)pow((double)c.beta2, (double)h->step_t));
+  }
+  // (bf16 path only: the fp32 debug path's GEMMs read the fp32 master weights,
+  // which the fused update would overwrite under a concurrent reader.)
+  const bool fused = h->bf != 0;
+  h->fuse_opt = fused;
+  r = backward_impl(h);
+  h->fuse_opt = false;
   if (r) return r;
-  r = fal_step(h);
-  if (r) return r;
+  const size_t blocks_begin = h->lp[0].w_qkv;
+  const bool bad = fused ? (adamw_range(h, 0, blocks_begin, blocks_begin) ||
+                            adamw_range(h, h->n_decay, h->n_params, h->n_decay))
+                         : adamw_range(h, 0, h->n_params, h->n_decay);
+  if (bad) return fail(h, FAL_ERR_CUDA, "AdamW launch failed");
+  h->sh_cur ^= 1;
+  h->state = 0;
   if (loss_host) {
     if (cudaMemcpyAsync(loss_host, h->loss, sizeof(float), cudaMemcpyDeviceToHost, h->sm) != cudaSuccess)
       return fail(h, FAL_ERR_CUDA, "loss copy failed");
@@ -877,7 +940,7 @@ int fal_set_params(fal_handle* h, const float* src, size_t n) {
   if (n != h->n_params) return fail(h, FAL_ERR_ARG, "parameter count mismatch");
   cudaStream_t s = h->sm;
   if (cudaMemcpyAsync(h->P, src, n * 4, cudaMemcpyDefault, s) != cudaSuccess) return fail(h, FAL_ERR_CUDA, "copy failed");
-  if (h->Sh && f32_to_bf16(n, h->P, h->Sh, s)) return fail(h, FAL_ERR_CUDA, "bf16 refresh failed");
+  if (h->bf && f32_to_bf16(n, h->P, h->Shb[h->sh_cur], s)) return fail(h, FAL_ERR_CUDA, "bf16 refresh failed");
   cudaMemsetAsync(h->Mo, 0, n * 4, s);
   cudaMemsetAsync(h->Vo, 0, n * 4, s);
   h->step_t = 0;

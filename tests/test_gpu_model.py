@@ -136,12 +136,14 @@ def test_call_order_errors():
     assert e.value.code == fal.FAL_ERR_STATE
 
 
-@pytest.mark.parametrize("variant,schedule", [("fal", "two_stream"), ("gpt", "serial"), ("falplus", "serial")])
-def test_fused_train_step_matches_separate_calls(variant, schedule):
-    """fal_train_step (one call for forward, backward and AdamW) leaves the
-    same parameters as forward + backward + step called one by one (up to the
-    reduction order of atomics in the gradients)."""
-    s = SMALL
+@pytest.mark.parametrize("variant,schedule,shape", [("fal", "two_stream", "small"), ("gpt", "serial", "small"),
+                                                    ("falplus", "serial", "small"), ("fal", "serial", "tiny")])
+def test_fused_train_step_matches_separate_calls(variant, schedule, shape):
+    """fal_train_step applies AdamW to the block matrices inside their
+    weight-gradient GEMMs; it must leave the same parameters (and gradients)
+    as forward + backward + step called one by one, up to the reduction order
+    of atomics in the gradients.  'tiny' runs the fp32 debug path."""
+    s = SMALL if shape == "small" else synth.SHAPES["tiny"].replace(layers=3)
     params = synth.perturb_params(synth.init_params(variant, s, 3), 3)
     tok, tgt = synth.make_tokens(s, 3)
     a, b = _model(variant, s, schedule), _model(variant, s, schedule)
@@ -154,8 +156,10 @@ def test_fused_train_step_matches_separate_calls(variant, schedule):
         b.step()
         assert abs(la - lb) <= 1e-6 * abs(lb)
     pa, pb = a.params(), b.params()
+    ga, gb = a.grads(), b.grads()
     for k in params:
         np.testing.assert_allclose(pa[k], pb[k], rtol=1e-5, atol=1e-7, err_msg=k)
+        np.testing.assert_allclose(ga[k], gb[k], rtol=1e-4, atol=1e-6, err_msg="d" + k)
 
 
 def test_training_reduces_loss():
