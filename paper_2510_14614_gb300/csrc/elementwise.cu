@@ -2,6 +2,8 @@
 // forward/backward (one warp per row, 128-bit vector access, warp-shuffle
 // reductions), column reductions for LN/bias gradients, the cross-entropy
 // head, and AdamW over the flat parameter buffer.
+#include <cstring>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -163,22 +165,24 @@ __global__ void __launch_bounds__(CS_COLS) colsum_kernel(ColsumArgs a) {
   a.partial[((long)chunk * 2 + 1) * a.d + c] = s1;
 }
 
-__global__ void colsum_finish_kernel(ColsumArgs a) {
+// Sums nchunk partials [nchunk][2][d]: slot 0 -> out0 (and out0b), slot 1 -> out1.
+__global__ void colsum_finish_kernel(const float* __restrict__ partial, int nchunk, int d, float* out1, float* out0,
+                                     float* out0b, int accumulate) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= a.d) return;
+  if (c >= d) return;
   float s0 = 0.f, s1 = 0.f;
-  for (int k = 0; k < CS_CHUNKS; ++k) {
-    s0 += a.partial[((long)k * 2 + 0) * a.d + c];
-    s1 += a.partial[((long)k * 2 + 1) * a.d + c];
+  for (int k = 0; k < nchunk; ++k) {
+    s0 += partial[((long)k * 2 + 0) * d + c];
+    s1 += partial[((long)k * 2 + 1) * d + c];
   }
-  if (a.accumulate) {
-    if (a.out0) a.out0[c] += s0;
-    if (a.out0b) a.out0b[c] += s0;
-    if (a.out1) a.out1[c] += s1;
+  if (accumulate) {
+    if (out0) out0[c] += s0;
+    if (out0b) out0b[c] += s0;
+    if (out1) out1[c] += s1;
   } else {
-    if (a.out0) a.out0[c] = s0;
-    if (a.out0b) a.out0b[c] = s0;
-    if (a.out1) a.out1[c] = s1;
+    if (out0) out0[c] = s0;
+    if (out0b) out0b[c] = s0;
+    if (out1) out1[c] = s1;
   }
 }
 
@@ -352,6 +356,10 @@ int last_err() { return cudaGetLastError() == cudaSuccess ? 0 : 4; }
 int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return 0;
   if (a.d % 4) return 1;
+  if (ln_fwd_bulk(act_bf16, a, s) == 0) {
+    count_launches(1);
+    return last_err();
+  }
   int r = act_bf16 ? ln_fwd_t<bf16>(a, s) : ln_fwd_t<float>(a, s);
   count_launches(1);
   return r ? r : last_err();
@@ -360,9 +368,30 @@ int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s) {
 int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return 0;
   if (a.d % 4) return 1;
+  if (ln_bwd_bulk(act_bf16, a, s) == 0) {
+    count_launches(a.cs_part ? 2 : 1);
+    return last_err();
+  }
   int r = act_bf16 ? ln_bwd_t<bf16>(a, s) : ln_bwd_t<float>(a, s);
   count_launches(1);
-  return r ? r : last_err();
+  if (r) return r;
+  if (a.cs_part) {
+    // column sums of the affine parameters' gradients by the separate reduction
+    ColsumArgs c;
+    memset(&c, 0, sizeof(c));
+    c.rows = a.rows; c.d = a.d; c.src = a.dy; c.src_act = 0; c.ld = a.d; c.src2 = a.dy2;
+    c.bmode = 1; c.x = a.x; c.mean = a.mean; c.rstd = a.rstd;
+    c.partial = a.cs_part; c.out1 = a.cs_out1; c.out0 = a.cs_out0; c.accumulate = a.cs_accumulate;
+    return colsum(act_bf16, c, s);
+  }
+  return last_err();
+}
+
+int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* out0, float* out0b, int accumulate,
+                  cudaStream_t s) {
+  if (d <= 0) return 0;
+  colsum_finish_kernel<<<(d + 255) / 256, 256, 0, s>>>(partial, nchunk, d, out1, out0, out0b, accumulate);
+  return last_err();
 }
 
 size_t colsum_partial_floats(int d) { return (size_t)CS_CHUNKS * 2 * d; }
@@ -372,7 +401,8 @@ int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
   dim3 grid((a.d + CS_COLS - 1) / CS_COLS, CS_CHUNKS);
   if (act_bf16) colsum_kernel<bf16><<<grid, CS_COLS, 0, s>>>(a);
   else colsum_kernel<float><<<grid, CS_COLS, 0, s>>>(a);
-  colsum_finish_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a);
+  colsum_finish_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a.partial, CS_CHUNKS, a.d, a.out1, a.out0, a.out0b,
+                                                          a.accumulate);
   count_launches(2);
   return last_err();
 }

@@ -81,6 +81,9 @@ struct LnFwdArgs {
   void* out2; const float* add_src; const float* add_g; const float* add_b;
 };
 int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s);
+// Sums nchunk per-chunk partial column sums [nchunk][2][d] into the outputs.
+int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* out0, float* out0b, int accumulate,
+                  cudaStream_t s);
 
 struct LnBwdArgs {
   int rows, d;
@@ -89,8 +92,17 @@ struct LnBwdArgs {
   const float* dres;                    // added to dx (residual branch), may be null
   float* dx;                            // fp32 out
   void* dx_act;                         // activation copy (may be null)
+  // Optional fused column sums of the affine parameters' gradients over the
+  // rows: cs_out1 (+)= sum (dy + dy2) * xhat, cs_out0 (+)= sum (dy + dy2).
+  // cs_part: scratch of colsum_partial_floats(d) floats.
+  float* cs_part; float* cs_out1; float* cs_out0; int cs_accumulate;
 };
 int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s);
+// Row-streaming LayerNorm kernels (one persistent CTA per SM, rows staged in
+// shared memory by bulk copies); 1 when the shape or alignment does not fit
+// them (the caller then uses the warp-per-row kernels).
+int ln_fwd_bulk(int act_bf16, const LnFwdArgs& a, cudaStream_t s);
+int ln_bwd_bulk(int act_bf16, const LnBwdArgs& a, cudaStream_t s);
 
 // Column sums over rows: s1[c] = sum_r a(r,c)*b(r,c), s0[c] = sum_r a(r,c)
 // with a = src (+ src2), b = LN-normalised x (bmode 1) or bsrc (bmode 2).

@@ -452,13 +452,17 @@ void ln_fwd_(Ctx& c, cudaStream_t s, const float* x, const float* gm, const floa
   c.check(ln_fwd(c.h->bf, a, s), "layernorm forward");
 }
 
+// LayerNorm backward; with dgamma/dbeta also the affine parameters' gradients
+// (column sums over the rows, computed in the same pass; part: scratch).
 void ln_bwd_(Ctx& c, cudaStream_t s, const float* dy, const float* dy2, const float* x, const float* mean,
-             const float* rstd, const float* gm, const float* dres, float* dx, void* dx_act) {
+             const float* rstd, const float* gm, const float* dres, float* dx, void* dx_act, float* part = nullptr,
+             float* dgamma = nullptr, float* dbeta = nullptr) {
   if (!c.ok()) return;
   LnBwdArgs a;
   memset(&a, 0, sizeof(a));
   a.rows = (int)c.h->BT; a.d = c.h->d; a.dy = dy; a.dy2 = dy2; a.x = x; a.mean = mean; a.rstd = rstd; a.gamma = gm;
   a.dres = dres; a.dx = dx; a.dx_act = dx_act;
+  if (dgamma || dbeta) { a.cs_part = part; a.cs_out1 = dgamma; a.cs_out0 = dbeta; }
   c.check(ln_bwd(c.h->bf, a, s), "layernorm backward");
 }
 
@@ -684,9 +688,8 @@ void layer_backward(Ctx& c, int i) {
             nullptr, 0);
     first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
     if (two) join(h);
-    ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act);
-    colsum_(c, s, h->part0, h->dU, 0, d, d, h->dU2, 1, A.X, A.ln1_mean, A.ln1_rstd, nullptr, Gp(h, p.ln1_g),
-            Gp(h, p.ln1_b), nullptr, 0);
+    ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
+            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
     return;
   }
   if (var == FAL_FAL) {  // block 1
@@ -695,16 +698,14 @@ void layer_backward(Ctx& c, int i) {
     // da_1 = dX_2 + (LN without affine)'(a_1) . dA1hat   (a_1 feeds X_2 and F)
     ln_bwd_(c, s, h->dA1hat, nullptr, h->a1, h->a1_mean, h->a1_rstd, nullptr, h->dX, h->dA, h->dA_act);
     attn_backward(c, i, h->dA, h->dA_act, s, h->part0, false);
-    ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act);
-    colsum_(c, s, h->part0, h->dU, 0, d, d, h->dU2, 1, A.X, A.ln1_mean, A.ln1_rstd, nullptr, Gp(h, p.ln1_g),
-            Gp(h, p.ln1_b), nullptr, 0);
+    ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
+            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
     return;
   }
   // GPT / FAL+
   mlp_backward(c, i, h->dX, h->dX_act, s, h->part0);
-  ln_bwd_(c, s, h->dU2, nullptr, A.Y, A.ln2_mean, A.ln2_rstd, Pp(h, p.ln2_g), h->dX, h->dY, h->dY_act);
-  colsum_(c, s, h->part0, h->dU2, 0, d, d, nullptr, 1, A.Y, A.ln2_mean, A.ln2_rstd, nullptr, Gp(h, p.ln2_g),
-          Gp(h, p.ln2_b), nullptr, 0);
+  ln_bwd_(c, s, h->dU2, nullptr, A.Y, A.ln2_mean, A.ln2_rstd, Pp(h, p.ln2_g), h->dX, h->dY, h->dY_act,
+          h->part0, Gp(h, p.ln2_g), Gp(h, p.ln2_b));
   const float* da = h->dY;
   const void* da_act = h->dY_act;
   if (var == FAL_FALPLUS && i >= 1) first_attention_grad(c, p.lnF_g, p.lnF_b, s, h->part0, 0);
@@ -714,9 +715,8 @@ void layer_backward(Ctx& c, int i) {
     da_act = h->dA_act;
   }
   attn_backward(c, i, da, da_act, s, h->part0, false);
-  ln_bwd_(c, s, h->dU, nullptr, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dY, h->dX, h->dX_act);
-  colsum_(c, s, h->part0, h->dU, 0, d, d, nullptr, 1, A.X, A.ln1_mean, A.ln1_rstd, nullptr, Gp(h, p.ln1_g),
-          Gp(h, p.ln1_b), nullptr, 0);
+  ln_bwd_(c, s, h->dU, nullptr, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dY, h->dX, h->dX_act,
+          h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
 }
 
 int backward_impl(fal_handle* h) {
@@ -728,9 +728,8 @@ int backward_impl(fal_handle* h) {
        "LM head dgrad");
   gemm(c, call1(h->V, d, seg(h->dlogits, h->Vp, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte), d, OUT_F32)), s,
        "LM head wgrad");
-  ln_bwd_(c, s, h->dU, nullptr, h->Xout, h->lnf_mean, h->lnf_rstd, Pp(h, h->lnf_g), nullptr, h->dX, h->dX_act);
-  colsum_(c, s, h->part0, h->dU, 0, d, d, nullptr, 1, h->Xout, h->lnf_mean, h->lnf_rstd, nullptr, Gp(h, h->lnf_g),
-          Gp(h, h->lnf_b), nullptr, 0);
+  ln_bwd_(c, s, h->dU, nullptr, h->Xout, h->lnf_mean, h->lnf_rstd, Pp(h, h->lnf_g), nullptr, h->dX, h->dX_act,
+          h->part0, Gp(h, h->lnf_g), Gp(h, h->lnf_b));
   if (h->cfg.variant != FAL_GPT) cudaMemsetAsync(h->dA1hat, 0, (size_t)BT * d * 4, s);
   if (h->cfg.variant == FAL_FAL) {
     cudaMemsetAsync(Gp(h, h->lnF_g), 0, (size_t)d * 4, s);
