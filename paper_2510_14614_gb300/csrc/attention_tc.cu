@@ -456,20 +456,25 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_tc_kernel(const __grid
       if (!mbar_wait(ps_ready, par, abort_flag)) { ok = false; break; }
       tc_fence_after();
       if (lane == 0) {
+        // dQ first, so that its read-out overlaps the dV / dK products
+#pragma unroll
+        for (int kk = 0; kk < 128 / 16; ++kk) {
+          const uint32_t b_mn = kk * 2048;  // MN-major [q or key rows][hd]
+          tc_mma(tmem + T_S, smem_desc(base + L::DS_OFF + b_mn, L::CHUNK, 1024),
+                 smem_desc(base + L::K_OFF + b_mn, L::CHUNK, 1024), id_q, kk > 0);
+        }
+        tc_commit(dq_full);
 #pragma unroll
         for (int kk = 0; kk < 128 / 16; ++kk) {
           const uint32_t a_k = (kk >> 2) * L::CHUNK + (kk & 3) * 32;  // K-major [keys][q] tiles
-          const uint32_t b_mn = kk * 2048;                             // MN-major [q or key rows][hd]
+          const uint32_t b_mn = kk * 2048;
           tc_mma(tmem + T_DV, smem_desc(base + L::P_OFF + a_k, 16, 1024),
                  smem_desc(base + L::DO_OFF + b_mn, L::CHUNK, 1024), id_kv, (it > 0 || kk > 0));
           tc_mma(tmem + T_DK, smem_desc(base + L::DS_OFF + a_k, 16, 1024),
                  smem_desc(base + L::Q_OFF + b_mn, L::CHUNK, 1024), id_kv, (it > 0 || kk > 0));
-          tc_mma(tmem + T_S, smem_desc(base + L::DS_OFF + b_mn, L::CHUNK, 1024),
-                 smem_desc(base + L::K_OFF + b_mn, L::CHUNK, 1024), id_q, kk > 0);
         }
         tc_commit(qdo_empty);
         tc_commit(ps_empty);
-        tc_commit(dq_full);
       }
       __syncwarp();
     }
@@ -494,16 +499,26 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_tc_kernel(const __grid
     const uint32_t lane_addr = tmem + ((uint32_t)(q4 * 32) << 16);
     const int tid = threadIdx.x - 64;  // 0..127
     bool ok = true;
+    // lse and D of the next query block travel in registers while the current
+    // block is processed, so their global latency stays off the critical path
+    float nl, nd;
+    {
+      const int t = kb * 128 + tid;
+      nl = (t < p.T) ? p.lse[(long)bh * p.T + t] : 0.f;
+      nd = (t < p.T) ? p.dvec[(long)bh * p.T + t] : 0.f;
+    }
     for (int it = 0; it < niter; ++it) {
       const uint32_t par = it & 1;
       const int q0 = (kb + it) * 128;
       named_sync_128(1);  // everyone is done with the previous block's lse / D
-      {
-        const int t = q0 + tid;
-        s_lse[tid] = (t < p.T) ? p.lse[(long)bh * p.T + t] : 0.f;
-        s_d[tid] = (t < p.T) ? p.dvec[(long)bh * p.T + t] : 0.f;
-      }
+      s_lse[tid] = nl;
+      s_d[tid] = nd;
       named_sync_128(1);
+      if (it + 1 < niter) {
+        const int t = q0 + 128 + tid;
+        nl = (t < p.T) ? p.lse[(long)bh * p.T + t] : 0.f;
+        nd = (t < p.T) ? p.dvec[(long)bh * p.T + t] : 0.f;
+      }
       if (!mbar_wait(sdp_full, par, abort_flag)) { ok = false; break; }
       if (!mbar_wait(ps_empty, par ^ 1u, abort_flag)) { ok = false; break; }
       tc_fence_after();

@@ -153,28 +153,60 @@ __global__ void __launch_bounds__(CS_COLS) colsum_kernel(ColsumArgs a) {
   const int r0 = chunk * per, r1 = min(a.rows, r0 + per);
   if (c >= a.d) return;
   float s0 = 0.f, s1 = 0.f;
-  for (int r = r0; r < r1; ++r) {
+  auto term = [&](int r) {
     float v = a.src_act ? to_f(reinterpret_cast<const act_t*>(a.src)[(long)r * a.ld + c])
                         : reinterpret_cast<const float*>(a.src)[(long)r * a.ld + c];
     if (a.src2) v += a.src2[(long)r * a.ld + c];
     s0 += v;
     if (a.bmode == 1) s1 += v * (a.x[(long)r * a.d + c] - a.mean[r]) * a.rstd[r];
     else if (a.bmode == 2) s1 += v * a.bsrc[(long)r * a.d + c];
+  };
+  // eight independent rows per step keep enough loads in flight per thread
+  int r = r0;
+  for (; r + 8 <= r1; r += 8) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) term(r + j);
   }
+  for (; r < r1; ++r) term(r);
   a.partial[((long)chunk * 2 + 0) * a.d + c] = s0;
   a.partial[((long)chunk * 2 + 1) * a.d + c] = s1;
 }
 
 // Sums nchunk partials [nchunk][2][d]: slot 0 -> out0 (and out0b), slot 1 -> out1.
-__global__ void colsum_finish_kernel(const float* __restrict__ partial, int nchunk, int d, float* out1, float* out0,
-                                     float* out0b, int accumulate) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= d) return;
+// One CTA per 32 columns: its 8 warps take every 8th chunk (one coalesced
+// 128-byte row segment per warp and slot), then combine through shared memory.
+constexpr int CF_WARPS = 8;
+__global__ void __launch_bounds__(CF_WARPS * 32) colsum_finish_kernel(const float* __restrict__ partial, int nchunk,
+                                                                      int d, float* out1, float* out0, float* out0b,
+                                                                      int accumulate) {
+  __shared__ float red[2][CF_WARPS][32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x * 32 + lane;
   float s0 = 0.f, s1 = 0.f;
-  for (int k = 0; k < nchunk; ++k) {
-    s0 += partial[((long)k * 2 + 0) * d + c];
-    s1 += partial[((long)k * 2 + 1) * d + c];
+  if (c < d) {
+    int k = warp;
+    for (; k + 3 * CF_WARPS < nchunk; k += 4 * CF_WARPS) {
+      float a[4], b[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        a[j] = partial[((long)(k + j * CF_WARPS) * 2 + 0) * d + c];
+        b[j] = partial[((long)(k + j * CF_WARPS) * 2 + 1) * d + c];
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) { s0 += a[j]; s1 += b[j]; }
+    }
+    for (; k < nchunk; k += CF_WARPS) {
+      s0 += partial[((long)k * 2 + 0) * d + c];
+      s1 += partial[((long)k * 2 + 1) * d + c];
+    }
   }
+  red[0][warp][lane] = s0;
+  red[1][warp][lane] = s1;
+  __syncthreads();
+  if (warp != 0 || c >= d) return;
+  s0 = s1 = 0.f;
+#pragma unroll
+  for (int w = 0; w < CF_WARPS; ++w) { s0 += red[0][w][lane]; s1 += red[1][w][lane]; }
   if (accumulate) {
     if (out0) out0[c] += s0;
     if (out0b) out0b[c] += s0;
@@ -390,7 +422,7 @@ int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
 int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* out0, float* out0b, int accumulate,
                   cudaStream_t s) {
   if (d <= 0) return 0;
-  colsum_finish_kernel<<<(d + 255) / 256, 256, 0, s>>>(partial, nchunk, d, out1, out0, out0b, accumulate);
+  colsum_finish_kernel<<<(d + 31) / 32, CF_WARPS * 32, 0, s>>>(partial, nchunk, d, out1, out0, out0b, accumulate);
   return last_err();
 }
 
@@ -401,8 +433,8 @@ int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
   dim3 grid((a.d + CS_COLS - 1) / CS_COLS, CS_CHUNKS);
   if (act_bf16) colsum_kernel<bf16><<<grid, CS_COLS, 0, s>>>(a);
   else colsum_kernel<float><<<grid, CS_COLS, 0, s>>>(a);
-  colsum_finish_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a.partial, CS_CHUNKS, a.d, a.out1, a.out0, a.out0b,
-                                                          a.accumulate);
+  colsum_finish_kernel<<<(a.d + 31) / 32, CF_WARPS * 32, 0, s>>>(a.partial, CS_CHUNKS, a.d, a.out1, a.out0, a.out0b,
+                                                                  a.accumulate);
   count_launches(2);
   return last_err();
 }
