@@ -148,6 +148,19 @@ typedef struct fal_profile {
 int fal_profile_enable(fal_handle* h, int enable);
 int fal_profile_read(fal_handle* h, fal_profile* out);
 
+/* Per-launch view of the same records (GEMM, attention, LayerNorm, column
+ * reductions, cross-entropy), in issue order, times in ms relative to the
+ * start of the first record; stream 0 is the main stream, 1 the side stream.
+ * kind: 0 GEMM, 1 attention forward, 2 attention backward, 3 other.
+ * Synchronizes; does not reset the records (fal_profile_read does).  Fills at
+ * most cap entries of the caller's array and sets *n to their count. */
+typedef struct fal_launch_record {
+    double start_ms, end_ms, flops;
+    int kind, stream;
+    char label[48];
+} fal_launch_record;
+int fal_profile_timeline(fal_handle* h, fal_launch_record* out, int cap, int* n);
+
 /* Number of kernels this library has launched in this process (all handles). */
 long long fal_launch_count(void);
 

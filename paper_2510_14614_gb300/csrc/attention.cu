@@ -17,7 +17,7 @@ namespace {
 constexpr float LOG2E = 1.4426950408889634f;
 
 // ------------------------------------------------------------ backward (bf16)
-// D[b,h,t] = sum_c dO[t,c] * O[t,c]; also clears the dQ accumulator.
+// D[b,h,t] = sum_c dO[t,c] * O[t,c]; also clears dq_acc when it is given.
 __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx,
                                     float* __restrict__ dvec, float* __restrict__ dq_acc, int T, int H, int hd) {
   const int warps = blockDim.x / 32;
@@ -33,20 +33,13 @@ __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __
   float acc = 0.f;
   for (int c = lane; c < hd; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(g[c]);
   acc = warp_sum(acc);
-  float* dq = dq_acc + (long)bt * d + h * hd;
-  for (int c = lane; c < hd; c += 32) dq[c] = 0.f;
+  if (dq_acc) {
+    float* dq = dq_acc + (long)bt * d + h * hd;
+    for (int c = lane; c < hd; c += 32) dq[c] = 0.f;
+  }
   if (lane == 0) {
     const int b = bt / T, t = bt % T;
     dvec[((long)b * H + h) * T + t] = acc;
-  }
-}
-
-__global__ void attn_bwd_post_kernel(const float* __restrict__ dq_acc, bf16* __restrict__ dqkv, long rows, int d) {
-  const long n = rows * d / 4;
-  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
-    const long e = i * 4;
-    const long r = e / d, c = e % d;
-    store4(dqkv + r * 3L * d + c, load4(dq_acc + e));
   }
 }
 
@@ -161,13 +154,12 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
     const int wpb = 4;
     dim3 pg((H + wpb - 1) / wpb, (unsigned)rows);
     attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx),
-                                               dvec, dq_acc, T, H, hd);
-    const int r = attn_bwd_tc(B, T, H, hd, qkv, dctx, lse, dvec, dq_acc, dqkv, dev_err, s, msg);
+                                               dvec, nullptr, T, H, hd);
+    count_launches(1);
+    const int r = attn_bwd2_tc(B, T, H, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
     if (r) return r;
-    const long n4 = rows * d / 4;
-    const int blocks = (int)((n4 + 255) / 256 < 4096 ? (n4 + 255) / 256 : 4096);
-    attn_bwd_post_kernel<<<blocks, 256, 0, s>>>(dq_acc, reinterpret_cast<bf16*>(dqkv), rows, d);
-    count_launches(2);
+    (void)dq_acc;
+    (void)d;
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
     zero_kv_grad<<<256, 256, 0, s>>>(reinterpret_cast<float*>(dqkv), rows, d);

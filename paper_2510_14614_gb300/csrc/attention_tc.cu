@@ -314,363 +314,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_fwd_tc_kernel(const __grid
   }
 }
 
-// ------------------------------------------------------------ backward
-// One CTA per (128-key block, head), looping over the 128-query blocks that can
-// see those keys (causal).  Per query block, with keys as TMEM lanes:
-//   S^T  = K Q^T, dP^T = V dO^T                (tcgen05, TMEM columns 0 / 128)
-//   P^T  = 2^(S^T*scale*log2e - lse[q]),  dS^T = P^T * (dP^T - D[q])
-//                                              (warps 2..5, one thread per key,
-//                                               bf16 tiles in shared memory)
-//   dV  += P^T dO,  dK += dS^T Q               (TMEM accumulators)
-//   dQ   = dS K  (dS^T read as an MN-major A)  (TMEM columns of S^T, freed)
-// Warps 6..9 (one thread per query) add dQ * scale into the fp32 dQ
-// accumulator with vector reductions; at the end warps 2..5 store dK * scale
-// and dV in bf16.  D = rowsum(dO * O) and the zeroed dQ accumulator come from
-// attn_bwd_pre_kernel, the bf16 dQ from attn_bwd_post_kernel.
-constexpr int AB_THREADS = 320;
-
-struct AttnBwdParams {
-  CUtensorMap qkv;   // [B*T, 3d] bf16, box 64 x 128, 128-byte swizzle
-  CUtensorMap dctx;  // [B*T, d]  bf16, box 64 x 128, 128-byte swizzle
-  const float* lse;  // [B, H, T]
-  const float* dvec; // [B, H, T]
-  float* dq_acc;     // [B*T, d] fp32
-  bf16* dqkv;        // [B*T, 3d]
-  int T, H, nkv;
-  float scale, scale_log2;
-  int* err;
-};
-
-template <int HD>
-struct AttnBwdSmem {
-  static constexpr int KCH = HD / 64;
-  static constexpr int CHUNK = 128 * 64 * 2;  // [128 rows][64] bf16
-  static constexpr int K_OFF = 0;
-  static constexpr int V_OFF = K_OFF + KCH * CHUNK;
-  static constexpr int Q_OFF = V_OFF + KCH * CHUNK;
-  static constexpr int DO_OFF = Q_OFF + KCH * CHUNK;
-  static constexpr int P_OFF = DO_OFF + KCH * CHUNK;   // P^T  [128 keys][128 q], two 64-q chunks
-  static constexpr int DS_OFF = P_OFF + 2 * CHUNK;     // dS^T [128 keys][128 q]
-  static constexpr int LSE_OFF = DS_OFF + 2 * CHUNK;   // 128 lse + 128 D (fp32)
-  static constexpr int BAR_OFF = LSE_OFF + 1024;
-  static constexpr int TOTAL = BAR_OFF + 256 + 1024;
-};
-
-__device__ __forceinline__ void named_sync_128(int id) {
-  asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory");
-}
-__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
-}
-
-template <int HD>
-__global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_tc_kernel(const __grid_constant__ AttnBwdParams p) {
-  using L = AttnBwdSmem<HD>;
-  constexpr int KCH = L::KCH;
-  extern __shared__ uint8_t smem_raw[];
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = (raw + 1023u) & ~1023u;
-  uint8_t* sbase = smem_raw + (base - raw);
-  const uint32_t bar = base + L::BAR_OFF;
-  const uint32_t kv_full = bar, qdo_full = bar + 8, qdo_empty = bar + 16, sdp_full = bar + 24, ps_ready = bar + 32,
-                 ps_empty = bar + 40, dq_full = bar + 48, dq_free = bar + 56, fin = bar + 64, drain = bar + 72;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sbase + L::BAR_OFF + 80);
-  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(sbase + L::BAR_OFF + 84);
-  float* s_lse = reinterpret_cast<float*>(sbase + L::LSE_OFF);
-  float* s_d = s_lse + 128;
-
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int kb = blockIdx.x;  // key block (block 0 sees the most query blocks: launched first)
-  const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
-  const int d = p.H * HD;
-  const int row_base = b * p.T;
-  const int key0 = kb * 128;
-  const int niter = p.nkv - kb;  // query blocks kb .. nkv-1
-
-  if (threadIdx.x == 0) {
-    mbar_init(kv_full, 1); mbar_init(qdo_full, 1); mbar_init(qdo_empty, 1); mbar_init(sdp_full, 1);
-    mbar_init(ps_ready, 4); mbar_init(ps_empty, 1); mbar_init(dq_full, 1); mbar_init(dq_free, 4);
-    mbar_init(fin, 1); mbar_init(drain, 1);
-    *abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  }
-  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), 512);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint32_t T_S = 0, T_DP = 128, T_DV = 256, T_DK = 256 + HD;  // TMEM column bases (dQ reuses T_S)
-
-  if (warp == 0) {
-    // ------------------------------------------------ producer
-    bool ok = true;
-    if (lane == 0) {
-      mbar_arrive_expect_tx(kv_full, 2 * KCH * L::CHUNK);
-      for (int c = 0; c < KCH; ++c) {
-        tma_load_2d(base + L::K_OFF + c * L::CHUNK, &p.qkv, d + h * HD + 64 * c, row_base + key0, kv_full);
-        tma_load_2d(base + L::V_OFF + c * L::CHUNK, &p.qkv, 2 * d + h * HD + 64 * c, row_base + key0, kv_full);
-      }
-    }
-    for (int it = 0; it < niter && ok; ++it) {
-      if (!mbar_wait(qdo_empty, (it & 1) ^ 1u, abort_flag)) { ok = false; break; }
-      if (lane == 0) {
-        const int q0 = (kb + it) * 128;
-        mbar_arrive_expect_tx(qdo_full, 2 * KCH * L::CHUNK);
-        for (int c = 0; c < KCH; ++c) {
-          tma_load_2d(base + L::Q_OFF + c * L::CHUNK, &p.qkv, h * HD + 64 * c, row_base + q0, qdo_full);
-          tma_load_2d(base + L::DO_OFF + c * L::CHUNK, &p.dctx, h * HD + 64 * c, row_base + q0, qdo_full);
-        }
-      }
-      __syncwarp();
-    }
-    if (!ok && lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
-  } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer
-    const uint32_t id_s = make_idesc_bf16(0, 0, 128, 128);   // S^T, dP^T
-    const uint32_t id_kv = make_idesc_bf16(0, 1, 128, HD);   // dV, dK: A K-major, B MN-major
-    const uint32_t id_q = make_idesc_bf16(1, 1, 128, HD);    // dQ: A (dS) and B (K) MN-major
-    bool ok = mbar_wait(kv_full, 0, abort_flag), issued = false;
-    for (int it = 0; it < niter && ok; ++it) {
-      const uint32_t par = it & 1;
-      if (!mbar_wait(qdo_full, par, abort_flag)) { ok = false; break; }
-      if (it > 0 && !mbar_wait(dq_free, par ^ 1u, abort_flag)) { ok = false; break; }
-      tc_fence_after();
-      if (lane == 0) {
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::CHUNK + (kk & 3) * 32;
-          tc_mma(tmem + T_S, smem_desc(base + L::K_OFF + off, 16, 1024), smem_desc(base + L::Q_OFF + off, 16, 1024),
-                 id_s, kk > 0);
-        }
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::CHUNK + (kk & 3) * 32;
-          tc_mma(tmem + T_DP, smem_desc(base + L::V_OFF + off, 16, 1024), smem_desc(base + L::DO_OFF + off, 16, 1024),
-                 id_s, kk > 0);
-        }
-        tc_commit(sdp_full);
-      }
-      __syncwarp();
-      issued = true;
-      if (!mbar_wait(ps_ready, par, abort_flag)) { ok = false; break; }
-      tc_fence_after();
-      if (lane == 0) {
-        // dQ first, so that its read-out overlaps the dV / dK products
-#pragma unroll
-        for (int kk = 0; kk < 128 / 16; ++kk) {
-          const uint32_t b_mn = kk * 2048;  // MN-major [q or key rows][hd]
-          tc_mma(tmem + T_S, smem_desc(base + L::DS_OFF + b_mn, L::CHUNK, 1024),
-                 smem_desc(base + L::K_OFF + b_mn, L::CHUNK, 1024), id_q, kk > 0);
-        }
-        tc_commit(dq_full);
-#pragma unroll
-        for (int kk = 0; kk < 128 / 16; ++kk) {
-          const uint32_t a_k = (kk >> 2) * L::CHUNK + (kk & 3) * 32;  // K-major [keys][q] tiles
-          const uint32_t b_mn = kk * 2048;
-          tc_mma(tmem + T_DV, smem_desc(base + L::P_OFF + a_k, 16, 1024),
-                 smem_desc(base + L::DO_OFF + b_mn, L::CHUNK, 1024), id_kv, (it > 0 || kk > 0));
-          tc_mma(tmem + T_DK, smem_desc(base + L::DS_OFF + a_k, 16, 1024),
-                 smem_desc(base + L::Q_OFF + b_mn, L::CHUNK, 1024), id_kv, (it > 0 || kk > 0));
-        }
-        tc_commit(qdo_empty);
-        tc_commit(ps_empty);
-      }
-      __syncwarp();
-    }
-    if (ok) {
-      if (lane == 0) tc_commit(fin);
-      __syncwarp();
-    } else {
-      if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
-      if (issued) {
-        if (lane == 0) tc_commit(drain);
-        __syncwarp();
-        const uint64_t t0 = global_timer_ns();
-        while (!mbar_try_wait(drain, 0) && global_timer_ns() - t0 < kWaitNs) {}
-      }
-      *abort_flag = 1;
-    }
-  } else if (warp < 6) {
-    // ------------------------------------------------ P^T and dS^T (one thread per key)
-    const int q4 = warp & 3;
-    const int r = q4 * 32 + lane;  // key row inside the block = TMEM lane
-    const int key = key0 + r;
-    const uint32_t lane_addr = tmem + ((uint32_t)(q4 * 32) << 16);
-    const int tid = threadIdx.x - 64;  // 0..127
-    bool ok = true;
-    // lse and D of the next query block travel in registers while the current
-    // block is processed, so their global latency stays off the critical path
-    float nl, nd;
-    {
-      const int t = kb * 128 + tid;
-      nl = (t < p.T) ? p.lse[(long)bh * p.T + t] : 0.f;
-      nd = (t < p.T) ? p.dvec[(long)bh * p.T + t] : 0.f;
-    }
-    for (int it = 0; it < niter; ++it) {
-      const uint32_t par = it & 1;
-      const int q0 = (kb + it) * 128;
-      named_sync_128(1);  // everyone is done with the previous block's lse / D
-      s_lse[tid] = nl;
-      s_d[tid] = nd;
-      named_sync_128(1);
-      if (it + 1 < niter) {
-        const int t = q0 + 128 + tid;
-        nl = (t < p.T) ? p.lse[(long)bh * p.T + t] : 0.f;
-        nd = (t < p.T) ? p.dvec[(long)bh * p.T + t] : 0.f;
-      }
-      if (!mbar_wait(sdp_full, par, abort_flag)) { ok = false; break; }
-      if (!mbar_wait(ps_empty, par ^ 1u, abort_flag)) { ok = false; break; }
-      tc_fence_after();
-      const bool diag = (kb + it) == kb;
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t sr[32], dr[32];
-        TMEM_LD32(lane_addr + T_S + c * 32, sr);
-        TMEM_LD32(lane_addr + T_DP + c * 32, dr);
-        tmem_wait_ld();
-        float pv[32], dv[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int ql = c * 32 + i, q = q0 + ql;
-          float pr = ex2_approx(__uint_as_float(sr[i]) * p.scale_log2 - s_lse[ql]);
-          const bool masked = q >= p.T || key >= p.T || (diag && q < key);
-          pr = masked ? 0.f : pr;
-          pv[i] = pr;
-          dv[i] = pr * (__uint_as_float(dr[i]) - s_d[ql]);
-        }
-        // two 16-byte granules of 8 queries each per 32-query chunk half ... 4 granules per chunk
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-          const int qg = c * 4 + g;           // granule index over 128 queries (8 queries each)
-          const int chunk = qg >> 3, gi = qg & 7;
-          const uint32_t off = chunk * L::CHUNK + r * 128 + ((gi ^ (r & 7)) << 4);
-          uint4 pk, dk;
-          __nv_bfloat162 a0 = __floats2bfloat162_rn(pv[g * 8], pv[g * 8 + 1]), a1 = __floats2bfloat162_rn(pv[g * 8 + 2], pv[g * 8 + 3]);
-          __nv_bfloat162 a2 = __floats2bfloat162_rn(pv[g * 8 + 4], pv[g * 8 + 5]), a3 = __floats2bfloat162_rn(pv[g * 8 + 6], pv[g * 8 + 7]);
-          pk.x = *reinterpret_cast<uint32_t*>(&a0); pk.y = *reinterpret_cast<uint32_t*>(&a1);
-          pk.z = *reinterpret_cast<uint32_t*>(&a2); pk.w = *reinterpret_cast<uint32_t*>(&a3);
-          __nv_bfloat162 b0 = __floats2bfloat162_rn(dv[g * 8], dv[g * 8 + 1]), b1 = __floats2bfloat162_rn(dv[g * 8 + 2], dv[g * 8 + 3]);
-          __nv_bfloat162 b2 = __floats2bfloat162_rn(dv[g * 8 + 4], dv[g * 8 + 5]), b3 = __floats2bfloat162_rn(dv[g * 8 + 6], dv[g * 8 + 7]);
-          dk.x = *reinterpret_cast<uint32_t*>(&b0); dk.y = *reinterpret_cast<uint32_t*>(&b1);
-          dk.z = *reinterpret_cast<uint32_t*>(&b2); dk.w = *reinterpret_cast<uint32_t*>(&b3);
-          *reinterpret_cast<uint4*>(sbase + L::P_OFF + off) = pk;
-          *reinterpret_cast<uint4*>(sbase + L::DS_OFF + off) = dk;
-        }
-      }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(ps_ready);
-    }
-    // dK (scaled) and dV rows of this key
-    if (ok && mbar_wait(fin, 0, abort_flag)) {
-      tc_fence_after();
-      bf16* dkp = p.dqkv + ((long)row_base + key) * 3L * d + d + h * HD;
-      bf16* dvp = dkp + d;
-#pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t kr[32], vr[32];
-        TMEM_LD32(lane_addr + T_DK + c * 32, kr);
-        TMEM_LD32(lane_addr + T_DV + c * 32, vr);
-        tmem_wait_ld();
-        if (key < p.T) {
-#pragma unroll
-          for (int i = 0; i < 32; i += 8) {
-            uint4 a, v;
-            __nv_bfloat162 x0 = __floats2bfloat162_rn(__uint_as_float(kr[i]) * p.scale, __uint_as_float(kr[i + 1]) * p.scale);
-            __nv_bfloat162 x1 = __floats2bfloat162_rn(__uint_as_float(kr[i + 2]) * p.scale, __uint_as_float(kr[i + 3]) * p.scale);
-            __nv_bfloat162 x2 = __floats2bfloat162_rn(__uint_as_float(kr[i + 4]) * p.scale, __uint_as_float(kr[i + 5]) * p.scale);
-            __nv_bfloat162 x3 = __floats2bfloat162_rn(__uint_as_float(kr[i + 6]) * p.scale, __uint_as_float(kr[i + 7]) * p.scale);
-            a.x = *reinterpret_cast<uint32_t*>(&x0); a.y = *reinterpret_cast<uint32_t*>(&x1);
-            a.z = *reinterpret_cast<uint32_t*>(&x2); a.w = *reinterpret_cast<uint32_t*>(&x3);
-            __nv_bfloat162 y0 = __floats2bfloat162_rn(__uint_as_float(vr[i]), __uint_as_float(vr[i + 1]));
-            __nv_bfloat162 y1 = __floats2bfloat162_rn(__uint_as_float(vr[i + 2]), __uint_as_float(vr[i + 3]));
-            __nv_bfloat162 y2 = __floats2bfloat162_rn(__uint_as_float(vr[i + 4]), __uint_as_float(vr[i + 5]));
-            __nv_bfloat162 y3 = __floats2bfloat162_rn(__uint_as_float(vr[i + 6]), __uint_as_float(vr[i + 7]));
-            v.x = *reinterpret_cast<uint32_t*>(&y0); v.y = *reinterpret_cast<uint32_t*>(&y1);
-            v.z = *reinterpret_cast<uint32_t*>(&y2); v.w = *reinterpret_cast<uint32_t*>(&y3);
-            *reinterpret_cast<uint4*>(dkp + c * 32 + i) = a;
-            *reinterpret_cast<uint4*>(dvp + c * 32 + i) = v;
-          }
-        }
-      }
-    } else if (lane == 0) {
-      set_dev_err(p.err, DEV_ERR_TIMEOUT);
-    }
-  } else {
-    // ------------------------------------------------ dQ read-out (one thread per query)
-    const int q4 = warp & 3;
-    const int r = q4 * 32 + lane;
-    const uint32_t lane_addr = tmem + ((uint32_t)(q4 * 32) << 16);
-    for (int it = 0; it < niter; ++it) {
-      const int q = (kb + it) * 128 + r;
-      if (!mbar_wait(dq_full, it & 1, abort_flag)) {
-        if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
-        break;
-      }
-      tc_fence_after();
-      float* dst = p.dq_acc + ((long)row_base + q) * d + h * HD;
-#pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t rr[32];
-        TMEM_LD32(lane_addr + T_S + c * 32, rr);
-        tmem_wait_ld();
-        if (q < p.T) {
-#pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            red_add_v4(dst + c * 32 + i, __uint_as_float(rr[i]) * p.scale, __uint_as_float(rr[i + 1]) * p.scale,
-                       __uint_as_float(rr[i + 2]) * p.scale, __uint_as_float(rr[i + 3]) * p.scale);
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(dq_free);
-    }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, 512);
-  }
-}
-
-template <int HD>
-int launch_bwd_tc(int B, int T, int H, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-                  float* dq_acc, void* dqkv, int* err, cudaStream_t s, std::string* msg) {
-  using L = AttnBwdSmem<HD>;
-  static bool set = false;
-  if (!set) {
-    if (cudaFuncSetAttribute(attn_bwd_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
-        cudaSuccess) {
-      if (msg) *msg = "attention backward smem attribute failed";
-      return 4;
-    }
-    set = true;
-  }
-  AttnBwdParams p;
-  memset(&p, 0, sizeof(p));
-  const long d = (long)H * HD;
-  if (!tma_map_2d(&p.qkv, qkv, 0, 3 * d, (unsigned long long)B * T, 3 * d, 64, 128, 1, msg)) return 1;
-  if (!tma_map_2d(&p.dctx, dctx, 0, d, (unsigned long long)B * T, d, 64, 128, 1, msg)) return 1;
-  p.lse = lse;
-  p.dvec = dvec;
-  p.dq_acc = dq_acc;
-  p.dqkv = reinterpret_cast<bf16*>(dqkv);
-  p.T = T;
-  p.H = H;
-  p.nkv = (T + 127) / 128;
-  p.scale = 1.f / sqrtf((float)HD);
-  p.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
-  p.err = err;
-  dim3 grid(p.nkv, B * H);
-  attn_bwd_tc_kernel<HD><<<grid, AB_THREADS, L::TOTAL, s>>>(p);
-  count_launches(1);
-  return 0;
-}
-
 template <int HD>
 int launch_fwd_tc(int B, int T, int H, const void* qkv, void* ctx, float* lse, int* err, cudaStream_t s,
                   std::string* msg) {
@@ -702,19 +345,6 @@ int launch_fwd_tc(int B, int T, int H, const void* qkv, void* ctx, float* lse, i
 }
 
 }  // namespace
-
-int attn_bwd_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-                float* dq_acc, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg) {
-  if (B <= 0 || T <= 0) return 0;
-  int r;
-  if (hd == 64) r = launch_bwd_tc<64>(B, T, H, qkv, dctx, lse, dvec, dq_acc, dqkv, dev_err, s, msg);
-  else if (hd == 128) r = launch_bwd_tc<128>(B, T, H, qkv, dctx, lse, dvec, dq_acc, dqkv, dev_err, s, msg);
-  else { if (msg) *msg = "tcgen05 attention needs head_dim 64 or 128"; return 6; }
-  if (r) return r;
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) { if (msg) *msg = std::string("attention backward launch: ") + cudaGetErrorString(e); return 4; }
-  return 0;
-}
 
 int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
                 std::string* msg) {

@@ -143,12 +143,13 @@ int num_sms();
 bool tma_map_2d(void* map128, const void* ptr, int f32, unsigned long long inner, unsigned long long outer,
                 unsigned long long ld, unsigned box_inner, unsigned box_outer, int swizzle128, std::string* msg);
 
-// tcgen05 flash-attention forward and backward main kernel (bf16, head_dim 64
-// or 128).  The backward expects dvec = rowsum(dO * O) and a zeroed dq_acc.
+// tcgen05 flash-attention forward (bf16, head_dim 64 or 128).
 int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
                 std::string* msg);
-int attn_bwd_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-                float* dq_acc, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
+// Two-pass tcgen05 attention backward (dK/dV per key block, then dQ per query
+// block, all accumulated in TMEM; no dQ accumulator).  dvec = rowsum(dO * O).
+int attn_bwd2_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
+                 void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
 
 // Process-wide count of kernel launches made by the library.
 void count_launches(long long n);

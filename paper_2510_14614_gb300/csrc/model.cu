@@ -107,7 +107,7 @@ struct fal_handle {
   size_t total_bytes = 0;
 
   // live kernel timing (fal_profile_enable)
-  struct ProfRec { cudaEvent_t a, b; int kind; double flops; };
+  struct ProfRec { cudaEvent_t a, b; int kind; double flops; const char* label; int stream; };
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_next = 0;
@@ -399,7 +399,9 @@ struct ProfScope {
   cudaEvent_t a = nullptr;
   int kind;
   double flops;
-  ProfScope(fal_handle* h_, cudaStream_t s_, int kind_, double flops_) : h(h_), s(s_), kind(kind_), flops(flops_) {
+  const char* label;
+  ProfScope(fal_handle* h_, cudaStream_t s_, int kind_, double flops_, const char* label_ = "")
+      : h(h_), s(s_), kind(kind_), flops(flops_), label(label_) {
     if (h->prof && (a = pool_event(h)) != nullptr) cudaEventRecord(a, s);
   }
   ~ProfScope() {
@@ -407,7 +409,7 @@ struct ProfScope {
     cudaEvent_t b = pool_event(h);
     if (!b) return;
     cudaEventRecord(b, s);
-    h->recs.push_back({a, b, kind, flops});
+    h->recs.push_back({a, b, kind, flops, label, s == h->sm ? 0 : 1});
   }
 };
 
@@ -422,7 +424,7 @@ void gemm(Ctx& c, const GemmCall& call, cudaStream_t s, const char* what) {
   if (!c.ok()) return;
   fal_handle* h = c.h;
   h->err.clear();
-  ProfScope ps(h, s, 0, gemm_flops(call));
+  ProfScope ps(h, s, 0, gemm_flops(call), what);
   int r = h->bf ? gemm_tc(call, h->dev_err, s, &h->err) : gemm_simt(call, 0, 0, s, &h->err);
   c.check(r, what);
 }
@@ -439,6 +441,7 @@ void colsum_(Ctx& c, cudaStream_t s, float* part, const void* src, int src_act, 
   a.rows = (int)h->BT; a.d = d; a.src = src; a.src_act = src_act; a.ld = ld; a.src2 = src2;
   a.bmode = bmode; a.x = x; a.mean = mean; a.rstd = rstd; a.bsrc = bsrc;
   a.partial = part; a.out1 = out1; a.out0 = out0; a.out0b = out0b; a.accumulate = accumulate;
+  ProfScope ps(h, s, 3, 0.0, "column reduction");
   c.check(colsum(h->bf, a, s), "column reduction");
 }
 
@@ -449,6 +452,7 @@ void ln_fwd_(Ctx& c, cudaStream_t s, const float* x, const float* gm, const floa
   memset(&a, 0, sizeof(a));
   a.rows = (int)c.h->BT; a.d = c.h->d; a.x = x; a.gamma = gm; a.beta = bt; a.out = out; a.out_f32 = out_f32;
   a.mean = mean; a.rstd = rstd; a.out2 = out2; a.add_src = add_src; a.add_g = add_g; a.add_b = add_b;
+  ProfScope ps(c.h, s, 3, 0.0, "layernorm forward");
   c.check(ln_fwd(c.h->bf, a, s), "layernorm forward");
 }
 
@@ -463,6 +467,7 @@ void ln_bwd_(Ctx& c, cudaStream_t s, const float* dy, const float* dy2, const fl
   a.rows = (int)c.h->BT; a.d = c.h->d; a.dy = dy; a.dy2 = dy2; a.x = x; a.mean = mean; a.rstd = rstd; a.gamma = gm;
   a.dres = dres; a.dx = dx; a.dx_act = dx_act;
   if (dgamma || dbeta) { a.cs_part = part; a.cs_out1 = dgamma; a.cs_out0 = dbeta; }
+  ProfScope ps(c.h, s, 3, 0.0, "layernorm backward");
   c.check(ln_bwd(c.h->bf, a, s), "layernorm backward");
 }
 
@@ -486,7 +491,7 @@ void qkv_and_attention(Ctx& c, int i, cudaStream_t s) {
   gemm(c, call1(BT, 3 * d, seg(A.u, d, 0, Wp(h, p.w_qkv), d, 0, d), e), s, "QKV projection");
   if (!c.ok()) return;
   h->err.clear();
-  ProfScope ps(h, s, 1, attn_fwd_flops(h));
+  ProfScope ps(h, s, 1, attn_fwd_flops(h), "attention forward");
   c.check(attn_fwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dev_err, s, &h->err), "attention forward");
 }
 
@@ -589,6 +594,7 @@ int forward_impl(fal_handle* h, const int32_t* tokens, const int32_t* targets) {
   // logits = xf wte^T (tied LM head), padded row pitch Vp
   gemm(c, call1((int)h->BT, h->V, seg(h->xf, h->d, 0, Wp(h, h->wte), h->d, 0, h->d), epi_out(h->logits, h->Vp, OUT_ACT)),
        s, "LM head");
+  ProfScope ps_ce(h, s, 3, 0.0, "cross-entropy");
   if (c.ok())
     c.check(cross_entropy(h->bf, (int)h->BT, h->V, h->Vp, h->logits, h->tgt, h->dlogits, h->loss_rows, h->loss,
                           h->dev_err, s),
@@ -638,7 +644,7 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   }
   if (!c.ok()) return;
   h->err.clear();
-  ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h));
+  ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
   c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dq_acc, h->dvec,
                    h->dev_err, s, &h->err),
           "attention backward");
@@ -653,7 +659,10 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
 void first_attention_grad(Ctx& c, size_t g_off, size_t b_off, cudaStream_t s, float* part, int accumulate) {
   fal_handle* h = c.h;
   if (!c.ok()) return;
-  c.check(add_scaled_cols((int)h->BT, h->d, h->dU2, Pp(h, g_off), h->dA1hat, s), "first-attention gradient");
+  {
+    ProfScope ps(h, s, 3, 0.0, "first-attention gradient");
+    c.check(add_scaled_cols((int)h->BT, h->d, h->dU2, Pp(h, g_off), h->dA1hat, s), "first-attention gradient");
+  }
   colsum_(c, s, part, h->dU2, 0, h->d, h->d, nullptr, 2, nullptr, nullptr, nullptr, h->a1hat, Gp(h, g_off), Gp(h, b_off),
           nullptr, accumulate);
 }
@@ -1011,6 +1020,26 @@ int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n
 int fal_profile_enable(fal_handle* h, int enable) {
   if (!h) return FAL_ERR_ARG;
   h->prof = enable != 0;
+  return FAL_OK;
+}
+
+int fal_profile_timeline(fal_handle* h, fal_launch_record* out, int cap, int* n) {
+  if (!h || !n || cap < 0 || (cap > 0 && !out)) return FAL_ERR_ARG;
+  *n = 0;
+  if (cudaStreamSynchronize(h->sm) != cudaSuccess || cudaStreamSynchronize(h->ss) != cudaSuccess)
+    return fail(h, FAL_ERR_CUDA, "synchronize failed");
+  if (h->recs.empty()) return FAL_OK;
+  const cudaEvent_t t0 = h->recs.front().a;
+  for (const auto& r : h->recs) {
+    if (*n >= cap) break;
+    fal_launch_record& o = out[*n];
+    memset(&o, 0, sizeof(o));
+    float a = 0.f, b = 0.f;
+    if (cudaEventElapsedTime(&a, t0, r.a) != cudaSuccess || cudaEventElapsedTime(&b, t0, r.b) != cudaSuccess) continue;
+    o.start_ms = a; o.end_ms = b; o.kind = r.kind; o.stream = r.stream; o.flops = r.flops;
+    snprintf(o.label, sizeof(o.label), "%s", r.label ? r.label : "");
+    ++*n;
+  }
   return FAL_OK;
 }
 

@@ -38,6 +38,11 @@ class FalProfile(ctypes.Structure):
                 ("attn_ms", ctypes.c_double), ("attn_flops", ctypes.c_double), ("attn_launches", ctypes.c_longlong)]
 
 
+class FalLaunchRecord(ctypes.Structure):
+    _fields_ = [("start_ms", ctypes.c_double), ("end_ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("kind", ctypes.c_int), ("stream", ctypes.c_int), ("label", ctypes.c_char * 48)]
+
+
 class FalError(RuntimeError):
     def __init__(self, code, msg):
         super().__init__(f"{msg} (status {code})")
@@ -65,6 +70,8 @@ _SIGS = {
     "fal_get_tap": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t]),
     "fal_profile_enable": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int]),
     "fal_profile_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(FalProfile)]),
+    "fal_profile_timeline": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(FalLaunchRecord), ctypes.c_int,
+                                            ctypes.POINTER(ctypes.c_int)]),
     "fal_launch_count": (ctypes.c_longlong, []),
     "fal_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
     "fal_status_string": (ctypes.c_char_p, [ctypes.c_int]),
@@ -237,6 +244,14 @@ class Model:
 
     def profile_enable(self, on=True):
         _check(lib().fal_profile_enable(self.h, int(on)), self.h, "fal_profile_enable")
+
+    def profile_timeline(self, cap=100000):
+        """Per-launch records since the last profile_read(): dicts with start/end ms, kind, stream, label."""
+        arr = (FalLaunchRecord * cap)()
+        n = ctypes.c_int(0)
+        _check(lib().fal_profile_timeline(self.h, arr, cap, ctypes.byref(n)), self.h, "fal_profile_timeline")
+        return [{"start_ms": r.start_ms, "end_ms": r.end_ms, "flops": r.flops, "kind": r.kind, "stream": r.stream,
+                 "label": r.label.decode()} for r in arr[:n.value]]
 
     def profile_read(self):
         p = FalProfile()
