@@ -41,7 +41,8 @@ int fal_kernel_attention_fwd(int B, int T, int H, int hd, const void* qkv, void*
 
 /* Backward of fal_kernel_attention_fwd: dqkv (bf16 [B*T, 3*H*hd]) from qkv,
  * ctx, lse and dctx (bf16 [B*T, H*hd]).  scratch: fp32 device buffer of at
- * least fal_kernel_attention_bwd_scratch(B, T, H, hd) floats (overwritten). */
+ * least fal_kernel_attention_bwd_scratch(B, T, H, hd) = B*H*T floats
+ * (overwritten: it receives D = rowsum(dO * O) per query and head). */
 size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd);
 int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
                              const void* dctx, void* dqkv, float* scratch, void* stream);
@@ -57,12 +58,12 @@ int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const
  * Scratch comes from one fixed array of FAL_NOALLOC_ATTN_SCRATCH_FLOATS fp32
  * values (16 MiB) compiled into libfal.so: every GPU that loads the library
  * holds it until the process exits.  The call needs
- * B*T*H*hd + B*H*T <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS and returns
+ * B*H*T <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS and returns
  * FAL_ERR_WORKSPACE (launching nothing) above that.  It never calls cudaMalloc,
  * cudaFree or any allocating routine.  The first call on each device looks up
  * the array's device address (cudaGetSymbolAddress, with that device current);
  * make that first call before any stream capture.  All calls share the one
- * array and each call clears what it needs, so calls that overlap on the GPU
+ * array and each call rewrites what it reads, so calls that overlap on the GPU
  * (different streams, or several host threads on one device) race: serialize
  * them. */
 #define FAL_NOALLOC_ATTN_SCRATCH_FLOATS (4u * 1024u * 1024u)

@@ -17,9 +17,9 @@ namespace {
 constexpr float LOG2E = 1.4426950408889634f;
 
 // ------------------------------------------------------------ backward (bf16)
-// D[b,h,t] = sum_c dO[t,c] * O[t,c]; also clears dq_acc when it is given.
+// D[b,h,t] = sum_c dO[t,c] * O[t,c].
 __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx,
-                                    float* __restrict__ dvec, float* __restrict__ dq_acc, int T, int H, int hd) {
+                                    float* __restrict__ dvec, int T, int H, int hd) {
   const int warps = blockDim.x / 32;
   const int w = blockIdx.x * warps + threadIdx.x / 32, lane = threadIdx.x % 32;
   const int d = H * hd;
@@ -33,10 +33,6 @@ __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __
   float acc = 0.f;
   for (int c = lane; c < hd; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(g[c]);
   acc = warp_sum(acc);
-  if (dq_acc) {
-    float* dq = dq_acc + (long)bt * d + h * hd;
-    for (int c = lane; c < hd; c += 32) dq[c] = 0.f;
-  }
   if (lane == 0) {
     const int b = bt / T, t = bt % T;
     dvec[((long)b * H + h) * T + t] = acc;
@@ -145,7 +141,7 @@ int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* c
 }
 
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
-             const void* dctx, void* dqkv, float* dq_acc, float* dvec, int* dev_err, cudaStream_t s, std::string* msg) {
+             const void* dctx, void* dqkv, float* dvec, int* dev_err, cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
   const long rows = (long)B * T;
   const int d = H * hd;
@@ -154,11 +150,10 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
     const int wpb = 4;
     dim3 pg((H + wpb - 1) / wpb, (unsigned)rows);
     attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx),
-                                               dvec, nullptr, T, H, hd);
+                                               dvec, T, H, hd);
     count_launches(1);
     const int r = attn_bwd2_tc(B, T, H, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
     if (r) return r;
-    (void)dq_acc;
     (void)d;
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
@@ -213,16 +208,15 @@ int noalloc_scratch(float** out) {
 extern "C" int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, const void* qkv, const void* ctx,
                                                 const float* lse, const void* dctx, void* dqkv, void* stream) {
   if (B < 0 || T < 0 || H <= 0 || hd <= 0 || !qkv || !ctx || !lse || !dctx || !dqkv) return FAL_ERR_ARG;
-  const size_t dq_floats = (size_t)B * T * H * hd;
-  const size_t need = dq_floats + (size_t)B * H * T;
+  const size_t need = (size_t)B * H * T;
   if (need > kNoAllocFloats) return FAL_ERR_WORKSPACE;
   float* scratch = nullptr;
   const int rc = noalloc_scratch(&scratch);
   if (rc != FAL_OK) return rc;
   std::string msg;
-  // attn_bwd's first kernel zeroes the dQ accumulator and writes every D entry,
-  // so nothing left in the shared array by an earlier call leaks into this one.
-  const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, scratch + dq_floats, nullptr,
+  // attn_bwd's first kernel writes every D entry before it is read, so nothing
+  // left in the shared array by an earlier call leaks into this one.
+  const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, nullptr,
                               reinterpret_cast<cudaStream_t>(stream), &msg);
   return r == 0 ? FAL_OK : r == 1 ? FAL_ERR_ARG : r == 6 ? FAL_ERR_UNSUPPORTED : FAL_ERR_CUDA;
 }

@@ -64,9 +64,9 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
 // fp32 debug: one thread per query row.
 int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
              cudaStream_t s, std::string* msg);
-// dq_acc: fp32 [B*T, H*hd] scratch, dvec: fp32 [B, H, T] scratch.
+// dvec: fp32 [B, H, T] scratch (receives D = rowsum(dO * O)).
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
-             const float* lse, const void* dctx, void* dqkv, float* dq_acc, float* dvec, int* dev_err,
+             const float* lse, const void* dctx, void* dqkv, float* dvec, int* dev_err,
              cudaStream_t s, std::string* msg);
 
 // ---------------------------------------------------------------- elementwise

@@ -50,16 +50,15 @@ int fal_kernel_attention_fwd(int B, int T, int H, int hd, const void* qkv, void*
 }
 
 size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd) {
-  return (size_t)B * T * H * hd + (size_t)B * H * T;
+  (void)hd;
+  return (size_t)B * H * T;
 }
 
 int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
                              const void* dctx, void* dqkv, float* scratch, void* stream) {
   if (B < 0 || T < 0 || H <= 0 || !qkv || !ctx || !lse || !dctx || !dqkv || !scratch) return FAL_ERR_ARG;
   std::string msg;
-  float* dq_acc = scratch;
-  float* dvec = scratch + (size_t)B * T * H * hd;
-  return map_rc(attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, dq_acc, dvec, nullptr,
+  return map_rc(attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, nullptr,
                          reinterpret_cast<cudaStream_t>(stream),
                          &msg));
 }

@@ -101,7 +101,7 @@ struct fal_handle {
   void *logits = nullptr, *dlogits = nullptr;
   float *dX = nullptr, *dY = nullptr, *dA = nullptr, *dU = nullptr, *dU2 = nullptr, *dA1hat = nullptr;
   void *dX_act = nullptr, *dY_act = nullptr, *dA_act = nullptr, *dctx = nullptr, *dh = nullptr, *dqkv = nullptr;
-  float *dq_acc = nullptr, *dvec = nullptr, *part0 = nullptr, *part1 = nullptr;
+  float *dvec = nullptr, *part0 = nullptr, *part1 = nullptr;
   float* stage = nullptr;
   size_t stage_floats = 0;
   size_t total_bytes = 0;
@@ -306,7 +306,6 @@ void carve(fal_handle* h, uint8_t* base) {
   h->dctx = b.take<uint8_t>(BT * d * a);
   h->dh = b.take<uint8_t>(BT * F * a);
   h->dqkv = b.take<uint8_t>(BT * 3 * d * a);
-  h->dq_acc = b.take<float>(BT * d);
   h->dvec = b.take<float>((size_t)h->B * h->H * h->T);
   const int cs_cols = 3 * h->d > h->F ? 3 * h->d : h->F;  // widest column reduction: b_qkv or b_up
   h->part0 = b.take<float>(colsum_partial_floats(cs_cols));
@@ -645,7 +644,7 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   if (!c.ok()) return;
   h->err.clear();
   ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
-  c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dq_acc, h->dvec,
+  c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dvec,
                    h->dev_err, s, &h->err),
           "attention backward");
   gemm(c, group_calls({call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), wgrad_out(h, p.w_qkv, d)),

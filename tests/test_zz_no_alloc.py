@@ -59,7 +59,7 @@ def test_noalloc_matches_allocating_entry_point_twice(B, T, H, hd):
 def test_noalloc_rejects_problems_above_its_fixed_scratch():
     import torch
     from paper_2510_14614_gb300 import fal
-    B, T, H, hd = 1, 8192, 8, 64  # B*T*H*hd = 4 Mi floats: together with D it exceeds the array
+    B, T, H, hd = 2, 65536, 64, 64  # D needs B*H*T = 8 Mi floats, twice the array
     dummy = torch.empty(16, dtype=torch.bfloat16, device="cuda")
     p = ctypes.c_void_p(dummy.data_ptr())
     code = fal.lib().fal_kernel_attention_bwd_noalloc(B, T, H, hd, p, p, p, p, p, None)
