@@ -133,9 +133,10 @@ int fal_get_grads(fal_handle* h, float* dst, size_t n);
  * stack output).  n must equal the tensor's element count (logits: B*T*V). */
 int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n);
 
-/* Live kernel timing for roofline reports.  While enabled, every GEMM and
- * attention launch of this handle is bracketed by CUDA events on its own
- * stream (no synchronization is added).  fal_profile_read() synchronizes,
+/* Live kernel timing for roofline reports.  While enabled (enable = 1), every
+ * GEMM and attention launch of this handle is bracketed by CUDA events on its
+ * own stream (no synchronization is added); enable = 2 brackets every launch
+ * (LayerNorm, column reductions, cross-entropy too) for fal_profile_timeline.  fal_profile_read() synchronizes,
  * sums the event intervals since the last read, and resets the counters.
  * FLOPs are algorithmic: 2*M*N*K per GEMM; causal attention counts half of
  * the dense 4*B*H*T^2*hd forward and twice that for the backward. */

@@ -108,7 +108,7 @@ struct fal_handle {
 
   // live kernel timing (fal_profile_enable)
   struct ProfRec { cudaEvent_t a, b; int kind; double flops; const char* label; int stream; };
-  bool prof = false;
+  int prof = 0;  // 0 off, 1 GEMM and attention launches, 2 every launch
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_next = 0;
   std::vector<ProfRec> recs;
@@ -401,7 +401,7 @@ struct ProfScope {
   const char* label;
   ProfScope(fal_handle* h_, cudaStream_t s_, int kind_, double flops_, const char* label_ = "")
       : h(h_), s(s_), kind(kind_), flops(flops_), label(label_) {
-    if (h->prof && (a = pool_event(h)) != nullptr) cudaEventRecord(a, s);
+    if (h->prof > (kind == 3 ? 1 : 0) && (a = pool_event(h)) != nullptr) cudaEventRecord(a, s);
   }
   ~ProfScope() {
     if (!a) return;
@@ -643,10 +643,12 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   }
   if (!c.ok()) return;
   h->err.clear();
-  ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
-  c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dvec,
-                   h->dev_err, s, &h->err),
-          "attention backward");
+  {
+    ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
+    c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dvec,
+                     h->dev_err, s, &h->err),
+            "attention backward");
+  }
   gemm(c, group_calls({call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), wgrad_out(h, p.w_qkv, d)),
                        call1(BT, d, dgrad_seg(h, h->dqkv, 3 * d, p.w_qkv, d), epi_out(h->dU, d, OUT_F32))}),
        s, "QKV wgrad + dgrad");
@@ -1018,7 +1020,7 @@ int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n
 
 int fal_profile_enable(fal_handle* h, int enable) {
   if (!h) return FAL_ERR_ARG;
-  h->prof = enable != 0;
+  h->prof = enable < 0 ? 0 : (enable > 2 ? 2 : enable);
   return FAL_OK;
 }
 
@@ -1051,7 +1053,7 @@ int fal_profile_read(fal_handle* h, fal_profile* out) {
     float ms = 0.f;
     if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) continue;
     if (r.kind == 0) { out->gemm_ms += ms; out->gemm_flops += r.flops; out->gemm_launches++; }
-    else { out->attn_ms += ms; out->attn_flops += r.flops; out->attn_launches++; }
+    else if (r.kind == 1 || r.kind == 2) { out->attn_ms += ms; out->attn_flops += r.flops; out->attn_launches++; }
   }
   h->recs.clear();
   h->ev_next = 0;

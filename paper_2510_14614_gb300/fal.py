@@ -242,8 +242,9 @@ class Model:
         _check(lib().fal_get_loss(self.h, ctypes.byref(v)), self.h, "fal_get_loss")
         return v.value
 
-    def profile_enable(self, on=True):
-        _check(lib().fal_profile_enable(self.h, int(on)), self.h, "fal_profile_enable")
+    def profile_enable(self, on=True, every_launch=False):
+        level = (2 if every_launch else 1) if on else 0
+        _check(lib().fal_profile_enable(self.h, level), self.h, "fal_profile_enable")
 
     def profile_timeline(self, cap=100000):
         """Per-launch records since the last profile_read(): dicts with start/end ms, kind, stream, label."""
