@@ -142,34 +142,133 @@ __global__ void __launch_bounds__(256) ln_bwd_kernel(LnBwdArgs a) {
 }
 
 // ------------------------------------------------------------ column sums
-constexpr int CS_COLS = 256;   // columns per block (one per thread)
-constexpr int CS_CHUNKS = 64;  // row chunks (partials)
+constexpr int CS_THREADS = 256;
+constexpr int CS_CHUNKS = 64;  // row chunks of the scalar fallback
 
-template <typename act_t>
-__global__ void __launch_bounds__(CS_COLS) colsum_kernel(ColsumArgs a) {
-  const int c = blockIdx.x * CS_COLS + threadIdx.x;
-  const int chunk = blockIdx.y;
-  const int per = (a.rows + CS_CHUNKS - 1) / CS_CHUNKS;
+// V consecutive values of row r from a [rows, ld] source of type T (fp32 or the
+// activation type), as floats.
+template <typename T, int V>
+__device__ __forceinline__ void load_row_vec(const T* p, float* v) {
+  if constexpr (V == 1) {
+    v[0] = to_f(p[0]);
+  } else if constexpr (sizeof(T) == 4) {
+#pragma unroll
+    for (int j = 0; j < V; j += 4) {
+      const float4 q = load4(reinterpret_cast<const float*>(p) + j);
+      v[j] = q.x; v[j + 1] = q.y; v[j + 2] = q.z; v[j + 3] = q.w;
+    }
+  } else {
+    // 8 bf16 per 16-byte load
+#pragma unroll
+    for (int j = 0; j < V; j += 8) {
+      const uint4 q = *reinterpret_cast<const uint4*>(p + j);
+      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[k]));
+        v[j + 2 * k] = f.x;
+        v[j + 2 * k + 1] = f.y;
+      }
+    }
+  }
+}
+
+// Per-chunk column sums: thread owns V consecutive columns, the CTA's y index
+// picks a range of rows; s0 = sum a, s1 = sum a*b (a = src (+ src2), b per bmode).
+// Rows are taken four at a time with every load issued before any is used.
+template <typename src_t, int V>
+__global__ void __launch_bounds__(CS_THREADS) colsum_kernel(ColsumArgs a) {
+  const int c = (blockIdx.x * CS_THREADS + threadIdx.x) * V;
+  const int chunk = blockIdx.y, nch = gridDim.y;
+  const int per = (a.rows + nch - 1) / nch;
   const int r0 = chunk * per, r1 = min(a.rows, r0 + per);
   if (c >= a.d) return;
-  float s0 = 0.f, s1 = 0.f;
-  auto term = [&](int r) {
-    float v = a.src_act ? to_f(reinterpret_cast<const act_t*>(a.src)[(long)r * a.ld + c])
-                        : reinterpret_cast<const float*>(a.src)[(long)r * a.ld + c];
-    if (a.src2) v += a.src2[(long)r * a.ld + c];
-    s0 += v;
-    if (a.bmode == 1) s1 += v * (a.x[(long)r * a.d + c] - a.mean[r]) * a.rstd[r];
-    else if (a.bmode == 2) s1 += v * a.bsrc[(long)r * a.d + c];
-  };
-  // eight independent rows per step keep enough loads in flight per thread
-  int r = r0;
-  for (; r + 8 <= r1; r += 8) {
+  const src_t* src = reinterpret_cast<const src_t*>(a.src);
+  float s0[V], s1[V];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) term(r + j);
+  for (int j = 0; j < V; ++j) s0[j] = s1[j] = 0.f;
+  auto rows4 = [&](int r, int n) {
+    float v[4][V], w[4][V], mu[4], rs[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (i >= n) continue;
+      load_row_vec<src_t, V>(src + (long)(r + i) * a.ld + c, v[i]);
+      if (a.src2) {
+        float t[V];
+        load_row_vec<float, V>(a.src2 + (long)(r + i) * a.ld + c, t);
+#pragma unroll
+        for (int j = 0; j < V; ++j) v[i][j] += t[j];
+      }
+      if (a.bmode == 1) {
+        load_row_vec<float, V>(a.x + (long)(r + i) * a.d + c, w[i]);
+        mu[i] = a.mean[r + i];
+        rs[i] = a.rstd[r + i];
+      } else if (a.bmode == 2) {
+        load_row_vec<float, V>(a.bsrc + (long)(r + i) * a.d + c, w[i]);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (i >= n) continue;
+#pragma unroll
+      for (int j = 0; j < V; ++j) {
+        s0[j] += v[i][j];
+        if (a.bmode == 1) s1[j] += v[i][j] * (w[i][j] - mu[i]) * rs[i];
+        else if (a.bmode == 2) s1[j] += v[i][j] * w[i][j];
+      }
+    }
+  };
+  int r = r0;
+  for (; r + 4 <= r1; r += 4) rows4(r, 4);
+  if (r < r1) rows4(r, r1 - r);
+#pragma unroll
+  for (int j = 0; j < V; ++j) {
+    a.partial[((long)chunk * 2 + 0) * a.d + c + j] = s0[j];
+    a.partial[((long)chunk * 2 + 1) * a.d + c + j] = s1[j];
   }
-  for (; r < r1; ++r) term(r);
-  a.partial[((long)chunk * 2 + 0) * a.d + c] = s0;
-  a.partial[((long)chunk * 2 + 1) * a.d + c] = s1;
+}
+
+// Plain column sums (no second source, no product term) over rows of 16-byte
+// segments: eight rows are requested before any is added, with the raw bytes
+// held in registers, so that ~1000 threads per SM keep ~128 KB in flight.
+template <typename src_t>
+__global__ void __launch_bounds__(CS_THREADS) colsum_plain_kernel(const src_t* __restrict__ src, long ld, int d,
+                                                                  int rows, float* __restrict__ partial) {
+  constexpr int V = 16 / (int)sizeof(src_t);
+  const int c = (blockIdx.x * CS_THREADS + threadIdx.x) * V;
+  const int chunk = blockIdx.y, nch = gridDim.y;
+  const int per = (rows + nch - 1) / nch;
+  const int r0 = chunk * per, r1 = min(rows, r0 + per);
+  if (c >= d) return;
+  float acc[V];
+#pragma unroll
+  for (int j = 0; j < V; ++j) acc[j] = 0.f;
+  for (int r = r0; r < r1; r += 8) {
+    uint4 q[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      q[i] = (r + i < r1) ? *reinterpret_cast<const uint4*>(src + (long)(r + i) * ld + c) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t w[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
+      if constexpr (sizeof(src_t) == 4) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc[k] += __uint_as_float(w[k]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[k]));
+          acc[2 * k] += f.x;
+          acc[2 * k + 1] += f.y;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < V; ++j) {
+    partial[((long)chunk * 2 + 0) * d + c + j] = acc[j];
+    partial[((long)chunk * 2 + 1) * d + c + j] = 0.f;
+  }
 }
 
 // Sums nchunk partials [nchunk][2][d]: slot 0 -> out0 (and out0b), slot 1 -> out1.
@@ -426,14 +525,39 @@ int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* o
   return last_err();
 }
 
-size_t colsum_partial_floats(int d) { return (size_t)CS_CHUNKS * 2 * d; }
+size_t colsum_partial_floats(int d) { return (size_t)kMaxColsumChunks * 2 * d; }
 
 int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
   if (a.d <= 0) return 0;
-  dim3 grid((a.d + CS_COLS - 1) / CS_COLS, CS_CHUNKS);
-  if (act_bf16) colsum_kernel<bf16><<<grid, CS_COLS, 0, s>>>(a);
-  else colsum_kernel<float><<<grid, CS_COLS, 0, s>>>(a);
-  colsum_finish_kernel<<<(a.d + 31) / 32, CF_WARPS * 32, 0, s>>>(a.partial, CS_CHUNKS, a.d, a.out1, a.out0, a.out0b,
+  // 16-byte row segments per thread when the layout allows (V = 8 bf16 or 4 fp32
+  // columns), else one column per thread; enough row chunks for ~3 CTAs per SM.
+  const bool src_bf16 = a.src_act && act_bf16;
+  const int vec = src_bf16 ? 8 : 4;
+  const bool aligned = (a.d % vec) == 0 && (a.ld % vec) == 0 && (!a.src2 || vec == 4 || (a.d % 4) == 0) &&
+                       (reinterpret_cast<uintptr_t>(a.src) & 15) == 0 &&
+                       (!a.src2 || (reinterpret_cast<uintptr_t>(a.src2) & 15) == 0) &&
+                       (!a.x || (reinterpret_cast<uintptr_t>(a.x) & 15) == 0) &&
+                       (!a.bsrc || (reinterpret_cast<uintptr_t>(a.bsrc) & 15) == 0);
+  const int V = aligned ? vec : 1;
+  const int col_blocks = (a.d / V + CS_THREADS - 1) / CS_THREADS;
+  int nch = aligned ? (3 * num_sms() + col_blocks - 1) / col_blocks : CS_CHUNKS;
+  if (nch > kMaxColsumChunks) nch = kMaxColsumChunks;
+  if (nch > a.rows) nch = a.rows > 0 ? a.rows : 1;
+  dim3 grid(col_blocks, nch);
+  if (aligned && a.bmode == 0 && !a.src2) {
+    if (src_bf16) colsum_plain_kernel<bf16><<<grid, CS_THREADS, 0, s>>>(reinterpret_cast<const bf16*>(a.src), a.ld, a.d,
+                                                                       a.rows, a.partial);
+    else colsum_plain_kernel<float><<<grid, CS_THREADS, 0, s>>>(reinterpret_cast<const float*>(a.src), a.ld, a.d,
+                                                               a.rows, a.partial);
+  } else if (!aligned) {
+    if (a.src_act && act_bf16) colsum_kernel<bf16, 1><<<grid, CS_THREADS, 0, s>>>(a);
+    else colsum_kernel<float, 1><<<grid, CS_THREADS, 0, s>>>(a);
+  } else if (src_bf16) {
+    colsum_kernel<bf16, 8><<<grid, CS_THREADS, 0, s>>>(a);
+  } else {
+    colsum_kernel<float, 4><<<grid, CS_THREADS, 0, s>>>(a);
+  }
+  colsum_finish_kernel<<<(a.d + 31) / 32, CF_WARPS * 32, 0, s>>>(a.partial, nch, a.d, a.out1, a.out0, a.out0b,
                                                                   a.accumulate);
   count_launches(2);
   return last_err();

@@ -98,7 +98,7 @@ struct LnBwdArgs {
   float* cs_part; float* cs_out1; float* cs_out0; int cs_accumulate;
 };
 int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s);
-// Row-streaming LayerNorm kernels (one persistent CTA per SM, rows staged in
+// Row-streaming LayerNorm kernels (two persistent CTAs per SM, rows staged in
 // shared memory by bulk copies); 1 when the shape or alignment does not fit
 // them (the caller then uses the warp-per-row kernels).
 int ln_fwd_bulk(int act_bf16, const LnFwdArgs& a, cudaStream_t s);
@@ -117,7 +117,8 @@ struct ColsumArgs {
   int accumulate;                 // add into destinations instead of storing
 };
 int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s);
-size_t colsum_partial_floats(int d);
+size_t colsum_partial_floats(int d);  // = kMaxColsumChunks * 2 * d
+constexpr int kMaxColsumChunks = 384;  // most per-chunk partials any column reduction writes
 
 int embed_fwd(int rows, int T, int d, int V, const int32_t* tok, const float* wte, const float* wpe,
               float* X, int* err, cudaStream_t s);

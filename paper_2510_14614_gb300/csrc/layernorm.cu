@@ -4,7 +4,7 @@
 //
 // These kernels are bound by HBM bandwidth.  Warp-per-row kernels that load a
 // row into registers keep too few bytes in flight per SM (every load holds an
-// L1 miss slot until it returns).  Here one persistent CTA per SM streams its
+// L1 miss slot until it returns).  Here persistent CTAs (two per SM) stream their
 // rows through a ring of shared-memory stages filled by bulk copies
 // (cp.async.bulk, issued by one producer thread, completion counted on an
 // mbarrier), so several rows per SM are always on their way from HBM without
@@ -17,7 +17,8 @@
 //
 // Every mbarrier wait is bounded; on expiry the CTA's consumers agree (barrier
 // reduction) to stop, the producer waits for the copies it issued, and the
-// launch returns normally.
+// launch returns normally.  Two CTAs share an SM, so that one CTA's row
+// reductions overlap the other's.
 #include "tc_ptx.cuh"
 
 namespace fal {
@@ -32,7 +33,7 @@ constexpr int LR_CONS = LR_WARPS * 32;      // consumer threads
 constexpr int LR_THREADS = LR_CONS + 32;    // + one producer warp
 constexpr int LR_MAX_D = 2 * 4 * LR_CONS;   // two 4-column groups per consumer thread
 constexpr int LR_MAX_STAGES = 8;
-constexpr uint32_t LR_STAGE_BUDGET = 192 * 1024;
+constexpr uint32_t LR_STAGE_BUDGET = 96 * 1024;  // two CTAs per SM
 constexpr uint32_t LR_TAIL_BYTES = 16 * LR_MAX_STAGES + 32 * 4 + 16;  // barriers, reduction slots, abort flag
 constexpr uint32_t LR_SMEM_MAX = LR_STAGE_BUDGET + LR_TAIL_BYTES;
 
@@ -96,7 +97,7 @@ __device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 
 
 // y = LN(x) (* gamma + beta); optional fp32 copy; out2 = y + add_src * add_g + add_b.
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 1) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes) {
+__global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
   volatile uint32_t* abort_flag;
@@ -186,7 +187,7 @@ __global__ void __launch_bounds__(LR_THREADS, 1) ln_fwd_rows_kernel(const LnFwdA
 // dx = rstd * (g - mean(g) - xhat * mean(g * xhat)) + dres with g = (dy + dy2) * gamma;
 // optional per-CTA column sums of (dy + dy2) * xhat and (dy + dy2).
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 1) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes) {
+__global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
   volatile uint32_t* abort_flag;
@@ -292,8 +293,8 @@ bool set_smem_attr(K kernel) {
 }
 
 int rows_grid(int rows) {
-  int g = num_sms();
-  if (g > 192) g = 192;  // per-CTA column partials must fit colsum_partial_floats(d)
+  int g = 2 * num_sms();
+  if (g > kMaxColsumChunks) g = kMaxColsumChunks;  // per-CTA column partials must fit colsum_partial_floats(d)
   return rows < g ? rows : g;
 }
 
