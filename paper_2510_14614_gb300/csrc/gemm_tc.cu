@@ -49,6 +49,11 @@ constexpr int TC_THREADS = 64 + 32 * TC_EPI_WARPS;
 
 struct TcGroup {
   int M, N, m_tiles, n_tiles, tile_start, nseg;
+  // Tile order: band_m = 0 walks m fastest over the whole group (the B panel of
+  // one column of tiles is read once; A must stay in L2).  band_m > 0 walks
+  // bands of band_m row tiles, each band across all column tiles, so that the
+  // CTAs in flight share their A rows and B stays in L2 (A is read once).
+  int band_m;
   int kb[2];
   int amap[2], bmap[2];
   int a_mn, b_mn;
@@ -272,6 +277,20 @@ __device__ __forceinline__ EpiOut epi_out_of(const TcGroup& G) {
   return o;
 }
 
+// Output tile (row index mt, column index nt) of a group-local tile index.
+__device__ __forceinline__ void tile_mn(const TcGroup& G, int local, int& mt, int& nt) {
+  if (G.band_m <= 0) {
+    mt = local % G.m_tiles;
+    nt = local / G.m_tiles;
+    return;
+  }
+  const int per_band = G.band_m * G.n_tiles;
+  const int band = local / per_band, r = local - band * per_band;
+  const int rows = min(G.band_m, G.m_tiles - band * G.band_m);  // the last band may be short
+  mt = band * G.band_m + r % rows;
+  nt = r / rows;
+}
+
 // Group of a tile index: groups own consecutive tile ranges in group order.
 __device__ __forceinline__ int group_of(const TcParams& p, int tile) {
   int g = 0;
@@ -287,9 +306,10 @@ template <bool MC>
 __device__ __forceinline__ void decode_tile(const TcParams& p, int tile, uint32_t rank, int& g, int& m0, int& n0) {
   g = group_of(p, tile);
   const TcGroup& G = p.grp[g];
-  const int local = tile - G.tile_start;
-  m0 = (local % G.m_tiles) * (MC ? 2 * TC_BM : TC_BM) + (int)rank * TC_BM;
-  n0 = (local / G.m_tiles) * TC_BN;
+  int mt, nt;
+  tile_mn(G, tile - G.tile_start, mt, nt);
+  m0 = mt * (MC ? 2 * TC_BM : TC_BM) + (int)rank * TC_BM;
+  n0 = nt * TC_BN;
 }
 
 // MC = true: launched in clusters of two CTAs on vertically adjacent tiles that
@@ -525,9 +545,10 @@ constexpr int T2_TILE = 256;
 __device__ __forceinline__ void decode_tile2(const TcParams& p, int tile, int& g, int& m0, int& n0) {
   g = group_of(p, tile);
   const TcGroup& G = p.grp[g];
-  const int local = tile - G.tile_start;
-  m0 = (local % G.m_tiles) * T2_TILE;
-  n0 = (local / G.m_tiles) * T2_TILE;
+  int mt, nt;
+  tile_mn(G, tile - G.tile_start, mt, nt);
+  m0 = mt * T2_TILE;
+  n0 = nt * T2_TILE;
 }
 
 template <typename act_t>
@@ -894,6 +915,12 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     T.m_tiles = (G.M + bm - 1) / bm;
     T.n_tiles = (G.N + bn - 1) / bn;
     T.tile_start = tiles;
+    {
+      // Bands of about one wave of tiles when a column of tiles is narrower
+      // than the machine: the A rows of a band are then read from DRAM once.
+      const int conc = pair ? pair_clusters : (mc ? mc_clusters : num_sms());
+      T.band_m = (T.n_tiles <= conc) ? (conc / T.n_tiles > 1 ? conc / T.n_tiles : 1) : 0;
+    }
     T.epi = G.epi;
     const EpiParams& e = G.epi;
     if (!check_ld(e.ldo, e.out) || !check_ld(e.ldo2, e.out2) || !check_ld(e.ldr, e.resid) ||
