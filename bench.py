@@ -87,6 +87,30 @@ def measured_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
+def gemm_traffic(workload, variant, schedule):
+    """DRAM bytes per tcgen05 GEMM launch from the committed ncu launch-list
+    summary of this workload (profiles/launches_<workload>_<variant>.md), or
+    None when there is none or when the GEMM sources changed since it was
+    captured (their SHA-256 is recorded next to the figure)."""
+    import hashlib
+    import re
+    if schedule != "two_stream":
+        return None
+    path = os.path.join(ROOT, "profiles", f"launches_{workload}_{variant}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    mb = re.search(r"^gemm_dram_bytes_per_launch:\s*(\d+)", text, re.M)
+    mh = re.search(r"^gemm_sources_sha256:\s*([0-9a-f]{64})", text, re.M)
+    if not mb or not mh:
+        return None
+    h = hashlib.sha256()
+    for f in ("gemm_tc.cu", "gemm_epi.cuh", "tc_ptx.cuh", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2510_14614_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return int(mb.group(1)) if h.hexdigest() == mh.group(1) else None
+
+
 # ------------------------------------------------------------------ oracle arm
 def oracle_step_sample(s, variant, seed=1234):
     """One fp64 oracle training step (forward, backward, AdamW) on a bounded
@@ -323,7 +347,10 @@ def main():
         "roofline": {
             "kernel": "gemm_tc_kernel (tcgen05 GEMM, all launches of the timed steps)",
             "bound": "tensor", "achieved": gemm_tflops, "peak": peak_sus, "unit": "TFLOP/s",
-            "frac": (gemm_tflops / peak_sus) if gemm_tflops else None, "traffic": None,
+            "frac": (gemm_tflops / peak_sus) if gemm_tflops else None,
+            "traffic": gemm_traffic(args.workload if args.layers is None and args.batch is None else "",
+                                    args.variant, args.schedule),
+            "traffic_unit": "DRAM bytes per launch (ncu launch list of this workload, profiles/)",
             "peak_kind": f"{peak_kind} bf16_tflops_sustained (kernel timed inside a long step)",
             "launches_per_step": prof["gemm_launches"] / args.steps,
             "time_share_of_step": prof["gemm_ms"] / (ms * args.steps),
