@@ -141,7 +141,8 @@ int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* c
 }
 
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
-             const void* dctx, void* dqkv, float* dvec, int* dev_err, cudaStream_t s, std::string* msg) {
+             const void* dctx, void* dqkv, float* dvec, int* dev_err, cudaStream_t s, std::string* msg,
+             int d_ready) {
   if (B <= 0 || T <= 0) return 0;
   const long rows = (long)B * T;
   const int d = H * hd;
@@ -149,9 +150,11 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
     if (hd != 64 && hd != 128) { if (msg) *msg = "bf16 attention needs head_dim 64 or 128"; return 6; }
     const int wpb = 4;
     dim3 pg((H + wpb - 1) / wpb, (unsigned)rows);
-    attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx),
-                                               dvec, T, H, hd);
-    count_launches(1);
+    if (!d_ready) {
+      attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx),
+                                                 reinterpret_cast<const bf16*>(dctx), dvec, T, H, hd);
+      count_launches(1);
+    }
     const int r = attn_bwd2_tc(B, T, H, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
     if (r) return r;
     (void)d;

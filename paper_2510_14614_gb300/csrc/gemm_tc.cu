@@ -252,6 +252,27 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep
   }
 }
 
+// Dot product of this lane's 32 output values (rounded to the activation type,
+// as stored) with the same 32 columns of rd_src: one head's share of D.
+template <typename act_t>
+__device__ __forceinline__ float rowdot_chunk(const EpiParams* ep, int M, int row, int col0, const uint32_t* r) {
+  if (row >= M) return 0.f;
+  const act_t* src = reinterpret_cast<const act_t*>(ep->rd_src) + (long)row * ep->rd_ld + col0;
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < 32; j += 4) {
+    const float4 o = load4(src + j);
+    s += to_f(from_f<act_t>(__uint_as_float(r[j]))) * o.x + to_f(from_f<act_t>(__uint_as_float(r[j + 1]))) * o.y +
+         to_f(from_f<act_t>(__uint_as_float(r[j + 2]))) * o.z + to_f(from_f<act_t>(__uint_as_float(r[j + 3]))) * o.w;
+  }
+  return s;
+}
+__device__ __forceinline__ void rowdot_store(const EpiParams* ep, int M, int row, int col_end, float s) {
+  if (row >= M) return;
+  const int T = ep->rd_T, h = (col_end - 1) / ep->rd_hd;
+  ep->rd_out[((long)(row / T) * ep->rd_H + h) * T + row % T] = s;
+}
+
 // Runs one chunk with the specialisation the group was prepared for.
 template <typename act_t>
 __device__ __forceinline__ void epi_chunk_dispatch(int kind, const TcParams& p, const EpiParams* ep, const EpiIn q,
@@ -499,6 +520,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       const int kind = G.kind;
       if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag)) break;
       tc_fence_after();
+      const bool rd = G.epi.rd_out != nullptr;
+      float rdot = 0.f;
       for (int c = 0; c < TC_BN / 64; ++c) {
         const int col0 = n0 + half * (TC_BN / 2) + c * 32;
         if (col0 >= eo.N) break;
@@ -507,6 +530,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
             tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2) + c * 32);
         TMEM_LD32(taddr, r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        if (rd) {
+          rdot += rowdot_chunk<act_t>(&G.epi, eo.M, m0 + q * 32 + lane, col0, r);
+          if ((col0 + 32) % G.epi.rd_hd == 0) { rowdot_store(&G.epi, eo.M, m0 + q * 32 + lane, col0 + 32, rdot); rdot = 0.f; }
+        }
         epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, m0 + q * 32, col0, r);
       }
       tc_fence_before();
@@ -709,6 +736,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       if (!mbar_wait_cluster(tfull_bar(acc), acc_phase, abort_flag)) break;
       tc_fence_after();
       const int row0 = m0 + (int)rank * 128 + q * 32;
+      const bool rd = G.epi.rd_out != nullptr;
+      float rdot = 0.f;
       for (int c = 0; c < TC_BN / 64; ++c) {
         const int col0 = n0 + half * (TC_BN / 2) + c * 32;
         if (col0 >= eo.N) break;
@@ -717,6 +746,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
             tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2) + c * 32);
         TMEM_LD32(taddr, r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        if (rd) {
+          rdot += rowdot_chunk<act_t>(&G.epi, eo.M, row0 + lane, col0, r);
+          if ((col0 + 32) % G.epi.rd_hd == 0) { rowdot_store(&G.epi, eo.M, row0 + lane, col0 + 32, rdot); rdot = 0.f; }
+        }
         epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, row0, col0, r);
       }
       tc_fence_before();
@@ -960,6 +993,12 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
       const bool special = k == 0 || k == EK_BIAS || k == (EK_BIAS | EK_GELU) || k == EK_DGELU ||
                            k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID) || k == EK_ADAMW;
       T.kind = special ? k : EK_ANY;
+    }
+    if (e.rd_out && (e.op != EPI_NONE || e.bias || e.bias2 || e.resid || e.resid2 || e.pre_f32 ||
+                     e.out_mode != OUT_ACT || e.rd_hd <= 0 || e.rd_hd % 32 || G.N % e.rd_hd || e.rd_T <= 0 ||
+                     e.rd_H <= 0 || !check_ld(e.rd_ld, e.rd_src) || (e.rd_ld & 7))) {
+      if (msg) *msg = "row-dot epilogue needs a plain activation output and head-aligned columns";
+      return 1;
     }
     if (e.op == EPI_ADAMW &&
         (e.out_mode != OUT_F32 || !e.opt_p || !e.opt_m || !e.opt_v || !check_ld(e.ldo, e.opt_p) ||

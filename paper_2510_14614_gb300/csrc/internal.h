@@ -38,6 +38,11 @@ struct EpiParams {
   // rbc2 are 1 / (1 - beta^t).
   float* opt_p; float* opt_m; float* opt_v; void* opt_sh;
   float opt_lr, opt_b1, opt_b2, opt_eps, opt_wd, opt_rbc1, opt_rbc2;
+  // Optional per-head row dot products of the (activation-rounded) output with
+  // rd_src (same [M, N] layout, row pitch rd_ld), for the attention backward's
+  // D = rowsum(dO * O): rd_out[((r / rd_T) * rd_H + c / rd_hd) * rd_T + r % rd_T]
+  // = sum over the head's columns c.  tcgen05 path only.
+  const void* rd_src; long rd_ld; float* rd_out; int rd_hd, rd_T, rd_H;
 };
 
 struct GemmOperand { const void* ptr; long ld; int mn_major; };
@@ -64,10 +69,11 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
 // fp32 debug: one thread per query row.
 int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
              cudaStream_t s, std::string* msg);
-// dvec: fp32 [B, H, T] scratch (receives D = rowsum(dO * O)).
+// dvec: fp32 [B, H, T] scratch (receives D = rowsum(dO * O)); d_ready: dvec
+// already holds D (computed by the GEMM that produced dctx).
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
              const float* lse, const void* dctx, void* dqkv, float* dvec, int* dev_err,
-             cudaStream_t s, std::string* msg);
+             cudaStream_t s, std::string* msg, int d_ready = 0);
 
 // ---------------------------------------------------------------- elementwise
 struct LnFwdArgs {

@@ -629,7 +629,8 @@ void mlp_backward(Ctx& c, int i, const float* dXn, const void* dXn_act, cudaStre
   colsum_(c, s, part, h->dh, 1, F, F, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_up), nullptr, 0);
 }
 
-void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStream_t s, float* part, bool skip_wo) {
+void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStream_t s, float* part, bool skip_wo,
+                   bool d_ready = false) {
   // dctx = da W_o; dW_o; db_o; attention backward; du = dqkv W_qkv -> dU; dW_qkv; db_qkv
   fal_handle* h = c.h;
   LayerA& A = h->la[i];
@@ -646,7 +647,7 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   {
     ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
     c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dvec,
-                     h->dev_err, s, &h->err),
+                     h->dev_err, s, &h->err, d_ready ? 1 : 0),
             "attention backward");
   }
   gemm(c, group_calls({call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), wgrad_out(h, p.w_qkv, d)),
@@ -680,9 +681,14 @@ void layer_backward(Ctx& c, int i) {
     // [dW_o | dW_down] = dX^T [ctx | g] and [dctx | dh] = dX [W_o | W_down] (dh with gelu').
     EpiParams edh = epi_out(h->dh, F, OUT_ACT);
     edh.op = EPI_DGELU; edh.aux = A.h; edh.ldx = F;
+    // dctx also yields the attention backward's D = rowsum(dctx * ctx) per head
+    EpiParams edc = epi_out(h->dctx, d, OUT_ACT);
+    if (h->bf) {
+      edc.rd_src = A.ctx; edc.rd_ld = d; edc.rd_out = h->dvec; edc.rd_hd = h->hd; edc.rd_T = h->T; edc.rd_H = h->H;
+    }
     gemm(c, group_calls({call1(d, d, wgrad_seg(h, h->dX_act, d, A.ctx, d), wgrad_out(h, p.w_o, d)),
                          call1(d, F, wgrad_seg(h, h->dX_act, d, A.g, F), wgrad_out(h, p.w_down, F)),
-                         call1(BT, d, dgrad_seg(h, h->dX_act, d, p.w_o, d), epi_out(h->dctx, d, OUT_ACT)),
+                         call1(BT, d, dgrad_seg(h, h->dX_act, d, p.w_o, d), edc),
                          call1(BT, F, dgrad_seg(h, h->dX_act, d, p.w_down, F), edh)}),
          s, "fused residual wgrad + dgrad");
     colsum_(c, s, h->part0, h->dX, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o),
@@ -690,7 +696,7 @@ void layer_backward(Ctx& c, int i) {
     const bool two = h->cfg.schedule == FAL_SCHED_TWO_STREAM && h->ss != h->sm;
     cudaStream_t sa = two ? h->ss : s;
     if (two) fork(h);
-    attn_backward(c, i, nullptr, nullptr, sa, two ? h->part1 : h->part0, true);
+    attn_backward(c, i, nullptr, nullptr, sa, two ? h->part1 : h->part0, true, h->bf != 0);
     gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), wgrad_out(h, p.w_up, d)),
                          call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
          s, "MLP up wgrad + dgrad");
