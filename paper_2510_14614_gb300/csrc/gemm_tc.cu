@@ -520,6 +520,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       const int kind = G.kind;
       if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag)) break;
       tc_fence_after();
+      int* ord_flag = G.epi.ord_role ? G.epi.ord_flags + (long)(tile - G.tile_start) * TC_EPI_WARPS + (warp - 2) : nullptr;
+      if (G.epi.ord_role == ORD_WAIT) {
+        // the same rows and columns of the signalling group must be in memory first
+        bool ok = true;
+        if (lane == 0) {
+          ok = flag_wait_eq(ord_flag, G.epi.ord_epoch, abort_flag);
+          fence_proxy_async_global();
+        }
+        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+          if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+          break;
+        }
+      }
       const bool rd = G.epi.rd_out != nullptr;
       float rdot = 0.f;
       for (int c = 0; c < TC_BN / 64; ++c) {
@@ -540,6 +553,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      if (G.epi.ord_role == ORD_SIGNAL) {
+        // publish this warp's 32 x 128 piece once its stores have landed
+        if (lane == 0) {
+          bulk_wait_all();
+          fence_proxy_async_global();
+          st_release_gpu(ord_flag, G.epi.ord_epoch);
+        }
+        __syncwarp();
+      }
     }
     if (lane == 0) bulk_wait_all();
     __syncwarp();
@@ -1024,6 +1046,37 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
       }
     }
     tiles += T.m_tiles * T.n_tiles;
+  }
+  // Groups of one launch that add into the same output must do so with TMA
+  // reduce-adds: the per-thread fallback is a plain read-modify-write.
+  for (int g = 0; g < c.ngroups; ++g)
+    for (int o = 0; o < c.ngroups; ++o)
+      if (o != g && p.grp[g].out_accum && !p.grp[g].out_tma && c.g[g].epi.out == c.g[o].epi.out) {
+        if (msg) *msg = "GEMM groups accumulating into one output need TMA-storable outputs";
+        return 1;
+      }
+  // Ordered split-K: every waiting group follows a signalling group of the same
+  // shape and output (its tiles come first in the static schedule, and tiles of
+  // a signalling group never wait, so every wait ends).
+  for (int g = 0; g < c.ngroups; ++g) {
+    const EpiParams& e = c.g[g].epi;
+    if (!e.ord_role) continue;
+    const TcGroup& T = p.grp[g];
+    bool ok = kind == TC_ONE && T.out_tma && e.ord_flags && e.ord_role >= ORD_SIGNAL && e.ord_role <= ORD_WAIT &&
+              (long)T.m_tiles * T.n_tiles * TC_EPI_WARPS <= (long)e.ord_cap && e.rd_out == nullptr;
+    if (ok && e.ord_role == ORD_WAIT) {
+      ok = false;
+      if (e.out_mode == OUT_F32_ACCUM)
+        for (int o = 0; o < g; ++o)
+          if (c.g[o].epi.ord_role == ORD_SIGNAL && c.g[o].epi.ord_flags == e.ord_flags &&
+              c.g[o].epi.ord_epoch == e.ord_epoch && c.g[o].epi.out == e.out && c.g[o].M == c.g[g].M &&
+              c.g[o].N == c.g[g].N)
+            ok = true;
+    }
+    if (!ok) {
+      if (msg) *msg = "ordered split-K needs the one-CTA engine, TMA outputs and a matching signalling group first";
+      return 1;
+    }
   }
   p.total_tiles = tiles;
   p.err = dev_err;

@@ -43,7 +43,15 @@ struct EpiParams {
   // D = rowsum(dO * O): rd_out[((r / rd_T) * rd_H + c / rd_hd) * rd_T + r % rd_T]
   // = sum over the head's columns c.  tcgen05 path only.
   const void* rd_src; long rd_ld; float* rd_out; int rd_hd, rd_T, rd_H;
+  // Ordered split-K over one output (tcgen05 one-CTA engine, TMA outputs):
+  // an ORD_SIGNAL group stores its tiles and then publishes, per tile and
+  // epilogue warp, ord_flags[...] = ord_epoch; a later ORD_WAIT group of the
+  // same launch and shape (OUT_F32_ACCUM) waits for that flag before it adds
+  // its partial, so the sum is formed in a fixed order.  ord_cap: ints in
+  // ord_flags; ord_epoch must differ from every value left by earlier launches.
+  int ord_role; int* ord_flags; int ord_cap; int ord_epoch;
 };
+enum OrdRole { ORD_NONE = 0, ORD_SIGNAL = 1, ORD_WAIT = 2 };
 
 struct GemmOperand { const void* ptr; long ld; int mn_major; };
 struct GemmSeg { GemmOperand A, B; int K; };

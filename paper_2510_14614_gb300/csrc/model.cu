@@ -18,6 +18,7 @@
 #include <cstring>
 #include <string>
 #include <initializer_list>
+#include <climits>
 #include <vector>
 
 #include "../../include/fal.h"
@@ -92,6 +93,9 @@ struct fal_handle {
   int sh_cur = 0;
   int32_t *tok = nullptr, *tgt = nullptr;
   int* dev_err = nullptr;
+  // per-tile flags of the ordered split-K residual GEMM; one new epoch per launch
+  int* ord_flags = nullptr;
+  int ord_cap = 0, ord_epoch = 0;
   float *loss = nullptr, *loss_rows = nullptr;
   std::vector<LayerA> la;
   float* Xout = nullptr;
@@ -263,6 +267,8 @@ void carve(fal_handle* h, uint8_t* base) {
   h->tok = b.take<int32_t>(BT);
   h->tgt = b.take<int32_t>(BT);
   h->dev_err = b.take<int>(4);
+  h->ord_cap = (int)(((BT + 127) / 128) * (((long)d + 255) / 256) * 8);
+  h->ord_flags = b.take<int>(h->ord_cap);
   h->loss = b.take<float>(4);
   h->loss_rows = b.take<float>(BT);
   h->la.assign(h->L, LayerA());
@@ -503,6 +509,14 @@ void up_gemm(Ctx& c, int i, cudaStream_t s) {
   gemm(c, call1((int)h->BT, h->F, seg(A.m, h->d, 0, Wp(h, p.w_up), h->d, 0, h->d), e), s, "MLP up-projection");
 }
 
+// Whether splitting an M x N output of 128 x 256 tiles in two halves of K fills
+// the last wave of the persistent grid (one CTA per SM) clearly better.
+bool split_k_pays(long M, long N) {
+  const long sms = num_sms(), tiles = ((M + 127) / 128) * ((N + 255) / 256);
+  auto fill = [&](long t) { return (double)t / (double)(((t + sms - 1) / sms) * sms); };
+  return fill(2 * tiles) > fill(tiles) + 0.05;
+}
+
 void layer_forward(Ctx& c, int i) {
   fal_handle* h = c.h;
   LayerA& A = h->la[i];
@@ -536,6 +550,26 @@ void layer_forward(Ctx& c, int i) {
     G.epi = epi_out(Xn, d, OUT_F32);
     G.epi.bias = Pp(h, p.b_o); G.epi.bias2 = Pp(h, p.b_down);
     G.epi.resid = A.X; G.epi.ldr = d;
+    if (h->bf && d % 64 == 0 && F > d && split_k_pays(BT, d)) {
+      // Two halves of K as two groups: twice the tiles of one N = d output, so
+      // the last wave of the persistent grid is nearly full.  The first half
+      // stores X_i + biases + its partial; the second adds its partial with TMA
+      // reduce-adds only after the same tile of the first half has landed, so
+      // the sum is formed in a fixed order (bitwise reproducible).
+      const int k1 = ((d + F) / 2 + 63) / 64 * 64 - d;
+      call.ngroups = 2;
+      G.seg[1].K = k1;
+      G.epi.ord_role = ORD_SIGNAL; G.epi.ord_flags = h->ord_flags; G.epi.ord_cap = h->ord_cap;
+      h->ord_epoch = h->ord_epoch == INT_MAX ? 1 : h->ord_epoch + 1;
+      G.epi.ord_epoch = h->ord_epoch;
+      GemmGroupDesc& G1 = call.g[1];
+      G1.M = BT; G1.N = d; G1.nseg = 1;
+      G1.seg[0] = seg((const uint8_t*)A.g + (size_t)k1 * h->asz, F, 0, (const uint8_t*)Wp(h, p.w_down) + (size_t)k1 * 2,
+                      F, 0, F - k1);
+      G1.epi = epi_out(Xn, d, OUT_F32_ACCUM);
+      G1.epi.ord_role = ORD_WAIT; G1.epi.ord_flags = h->ord_flags; G1.epi.ord_cap = h->ord_cap;
+      G1.epi.ord_epoch = G.epi.ord_epoch;
+    }
     gemm(c, call, s, "fused residual GEMM");
     return;
   }
@@ -822,6 +856,7 @@ int fal_create(const fal_config* cfg, void* workspace, size_t bytes, void* strea
   for (void* b : h->Shb)
     if (b) cudaMemsetAsync(b, 0, h->n_params * 2, s);
   cudaMemsetAsync(h->dev_err, 0, 16, s);
+  cudaMemsetAsync(h->ord_flags, 0, (size_t)h->ord_cap * sizeof(int), s);
   if (cudaStreamSynchronize(s) != cudaSuccess) {
     cudaEventDestroy(h->ev_fork);
     cudaEventDestroy(h->ev_join);

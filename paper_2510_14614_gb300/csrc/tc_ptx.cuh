@@ -221,6 +221,26 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+// Orders this thread's async-proxy (TMA) global accesses with its generic ones.
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+__device__ __forceinline__ void st_release_gpu(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Bounded wait for a global flag written by another CTA of the same launch.
+__device__ __forceinline__ bool flag_wait_eq(const int* f, int v, volatile uint32_t* abort_flag) {
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (ld_acquire_gpu(f) == v) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > kWaitNs) { *abort_flag = 1; return false; }
+    __nanosleep(64);
+  }
+}
 
 // TMEM store, 32 lanes x 32 columns (one register per column), and its wait.
 #define TMEM_ST32(taddr, r)                                                                          \

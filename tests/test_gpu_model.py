@@ -136,14 +136,20 @@ def test_call_order_errors():
     assert e.value.code == fal.FAL_ERR_STATE
 
 
+# GPT-2-small width at depth 3, one sequence: the FAL residual GEMM of blocks 2
+# and 3 (24 output tiles of 128 x 256) runs as two ordered halves of K.
+SPLITK = synth.SHAPES["gpt2_small"].replace(layers=3, batch=1)
+
+
 @pytest.mark.parametrize("variant,schedule,shape", [("fal", "two_stream", "small"), ("gpt", "serial", "small"),
-                                                    ("falplus", "serial", "small"), ("fal", "serial", "tiny")])
+                                                    ("falplus", "serial", "small"), ("fal", "serial", "tiny"),
+                                                    ("fal", "two_stream", "splitk")])
 def test_fused_train_step_matches_separate_calls(variant, schedule, shape):
     """fal_train_step applies AdamW to the block matrices inside their
     weight-gradient GEMMs; it must leave the same parameters (and gradients)
     as forward + backward + step called one by one, up to the reduction order
     of atomics in the gradients.  'tiny' runs the fp32 debug path."""
-    s = SMALL if shape == "small" else synth.SHAPES["tiny"].replace(layers=3)
+    s = {"small": SMALL, "splitk": SPLITK}.get(shape) or synth.SHAPES["tiny"].replace(layers=3)
     params = synth.perturb_params(synth.init_params(variant, s, 3), 3)
     tok, tgt = synth.make_tokens(s, 3)
     a, b = _model(variant, s, schedule), _model(variant, s, schedule)
@@ -171,3 +177,17 @@ def test_training_reduces_loss():
     losses = [m.train_step(tok, tgt) for _ in range(6)]
     assert losses[-1] < losses[0]
     assert m.loss() == losses[-1]  # the last forward's loss stays readable after the step
+
+
+def test_split_k_residual_is_reproducible():
+    """The two halves of the split residual GEMM add into X_{i+1} in a fixed
+    order: two forward passes give bitwise identical residual streams."""
+    s = SPLITK
+    m = _model("fal", s)
+    m.set_params(synth.perturb_params(synth.init_params("fal", s, 1), 1))
+    tok, tgt = synth.make_tokens(s, 1)
+    m.forward(tok, tgt)
+    first = [m.tap("X", i).copy() for i in range(1, s.layers + 1)]
+    m.forward(tok, tgt)
+    for i, x in enumerate(first, start=1):
+        np.testing.assert_array_equal(m.tap("X", i), x, err_msg=f"X{i}")
