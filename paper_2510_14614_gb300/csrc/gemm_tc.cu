@@ -23,9 +23,15 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cstring>
+#include <functional>
+#include <map>
 #include <mutex>
+#include <queue>
+#include <utility>
+#include <vector>
 
 #include "gemm_epi.cuh"
 #include "tc_ptx.cuh"
@@ -72,7 +78,21 @@ struct TcParams {
   TcGroup grp[kMaxGemmGroups];
   int ngroups, total_tiles;
   int* err;
+  // Tile lists per unit (CTA, or cluster of two): sched[u] .. sched[u + 1] index
+  // the tiles of unit u in sched[nunits + 1 + ...].  Null: round robin, unit u
+  // takes tiles u, u + nunits, ...
+  const int* sched;
 };
+
+// The i-th tile of a unit's sequence, or -1 when the unit is done.
+__device__ __forceinline__ int tile_at(const TcParams& p, int unit, int nunits, int i) {
+  if (p.sched) {
+    const int b = __ldg(p.sched + unit), e = __ldg(p.sched + unit + 1);
+    return i < e - b ? __ldg(p.sched + nunits + 1 + b + i) : -1;
+  }
+  const int t = unit + i * nunits;
+  return t < p.total_tiles ? t : -1;
+}
 
 
 // One epilogue warp's 32x32 accumulator chunk (rows row0.., columns col0..),
@@ -387,7 +407,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     uint32_t phase = 0;
     uint32_t issued_mask = 0, issued_par = 0;
     bool ok = true;
-    for (int tile = unit; tile < p.total_tiles && ok; tile += nunits) {
+    for (int ti = 0, tile; ok && (tile = tile_at(p, unit, nunits, ti)) >= 0; ++ti) {
       int g, m0, n0;
       decode_tile<MC>(p, tile, rank, g, m0, n0);
       const TcGroup& G = p.grp[g];
@@ -463,7 +483,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true, issued_any = false;
-      for (int tile = unit; tile < p.total_tiles && ok; tile += nunits) {
+      for (int ti = 0, tile; ok && (tile = tile_at(p, unit, nunits, ti)) >= 0; ++ti) {
         const int g = group_of(p, tile);
         const TcGroup& G = p.grp[g];
         const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
@@ -511,7 +531,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     float4* stage = reinterpret_cast<float4*>(smem_raw + (stage_s - raw));
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = unit; tile < p.total_tiles; tile += nunits) {
+    for (int ti = 0, tile; (tile = tile_at(p, unit, nunits, ti)) >= 0; ++ti) {
       int g, m0, n0;
       decode_tile<MC>(p, tile, rank, g, m0, n0);
       const TcGroup& G = p.grp[g];
@@ -645,7 +665,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
     uint32_t phase = 0;
     uint32_t issued_mask = 0, issued_par = 0;
     bool ok = true;
-    for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
+    for (int ti = 0, tile; ok && (tile = tile_at(p, cluster_id, nclusters, ti)) >= 0; ++ti) {
       int g, m0, n0;
       decode_tile2(p, tile, g, m0, n0);
       const TcGroup& G = p.grp[g];
@@ -702,7 +722,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true, issued_any = false;
-      for (int tile = cluster_id; tile < p.total_tiles && ok; tile += nclusters) {
+      for (int ti = 0, tile; ok && (tile = tile_at(p, cluster_id, nclusters, ti)) >= 0; ++ti) {
         const int g = group_of(p, tile);
         const TcGroup& G = p.grp[g];
         const int nkb = G.kb[0] + (G.nseg > 1 ? G.kb[1] : 0);
@@ -748,7 +768,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
     float4* stage = reinterpret_cast<float4*>(smem_raw + (stage_s - raw));
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = cluster_id; tile < p.total_tiles; tile += nclusters) {
+    for (int ti = 0, tile; (tile = tile_at(p, cluster_id, nclusters, ti)) >= 0; ++ti) {
       int g, m0, n0;
       decode_tile2(p, tile, g, m0, n0);
       const TcGroup& G = p.grp[g];
@@ -939,6 +959,72 @@ int max_pair_clusters(K kernel, int smem) {
   return n;
 }
 
+// Longest-first assignment of tiles to the units of the persistent grid, for
+// launches whose groups differ in depth K (a weight-gradient group with
+// K = B*T beside data-gradient groups with K = d or d_ff).  Round robin gives
+// every unit the same number of tiles, so the units that draw more of the deep
+// ones finish last.  A tile costs its K plus a fixed pipeline overhead; tiles
+// go, deepest group first and in tile order within a group, to the unit with
+// the least work so far.  The lists live in device memory, built once per
+// (units, group tiles and depths) for the life of the process.  Launches with
+// an ordered split-K keep round robin: their waits rely on it.
+const int* tile_schedule(const GemmCall& c, const TcParams& p, int nunits) {
+  long depth[kMaxGemmGroups];
+  bool uneven = false;
+  for (int g = 0; g < c.ngroups; ++g) {
+    if (c.g[g].epi.ord_role) return nullptr;
+    depth[g] = 0;
+    for (int k = 0; k < c.g[g].nseg; ++k) depth[g] += c.g[g].seg[k].K;
+    uneven = uneven || depth[g] != depth[0];
+  }
+  if (!uneven || nunits <= 1) return nullptr;
+  std::vector<long> key = {nunits, c.ngroups};
+  for (int g = 0; g < c.ngroups; ++g) {
+    key.push_back((long)p.grp[g].m_tiles * p.grp[g].n_tiles);
+    key.push_back(depth[g]);
+  }
+  static std::mutex mu;
+  static std::map<std::vector<long>, int*> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int order[kMaxGemmGroups];
+  for (int g = 0; g < c.ngroups; ++g) order[g] = g;
+  std::stable_sort(order, order + c.ngroups, [&](int a, int b) { return depth[a] > depth[b]; });
+  typedef std::pair<long, int> Load;
+  std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
+  for (int u = 0; u < nunits; ++u) heap.push(Load(0, u));
+  std::vector<std::vector<int>> lists(nunits);
+  for (int oi = 0; oi < c.ngroups; ++oi) {
+    const TcGroup& G = p.grp[order[oi]];
+    const long cost = depth[order[oi]] + 384;
+    for (int t = G.tile_start; t < G.tile_start + G.m_tiles * G.n_tiles; ++t) {
+      Load l = heap.top();
+      heap.pop();
+      lists[l.second].push_back(t);
+      heap.push(Load(l.first + cost, l.second));
+    }
+  }
+  std::vector<int> flat(nunits + 1 + p.total_tiles), seen(p.total_tiles, 0);
+  int n = 0;
+  for (int u = 0; u < nunits; ++u) {
+    flat[u] = n;
+    for (int t : lists[u]) { flat[nunits + 1 + n++] = t; ++seen[t]; }
+  }
+  flat[nunits] = n;
+  for (int t = 0; t < p.total_tiles; ++t)
+    if (seen[t] != 1) return nullptr;  // cannot happen; round robin is always valid
+  int* d = nullptr;
+  if (cudaMalloc(&d, flat.size() * sizeof(int)) != cudaSuccess) { cudaGetLastError(); return nullptr; }
+  if (cudaMemcpy(d, flat.data(), flat.size() * sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(d);
+    return nullptr;
+  }
+  cache[key] = d;
+  return d;
+}
+
 int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, std::string* msg) {
   if (!get_encoder(msg)) return 4;
   static bool attr_set = false;
@@ -1081,11 +1167,14 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
   p.total_tiles = tiles;
   p.err = dev_err;
   if (tiles == 0) return 0;
+  const int cap = pair ? pair_clusters : (mc ? mc_clusters : num_sms());
+  const int nunits = tiles < cap ? tiles : cap;
+  p.sched = tile_schedule(c, p, nunits);
   if (pair) {
-    const int clusters = tiles < pair_clusters ? tiles : pair_clusters;
+    const int clusters = nunits;
     gemm_tc2_kernel<bf16><<<2 * clusters, TC_THREADS, T2_SMEM, s>>>(p);
   } else if (mc) {
-    const int clusters = tiles < mc_clusters ? tiles : mc_clusters;
+    const int clusters = nunits;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * clusters, 1, 1);
     cfg.blockDim = dim3(TC_THREADS, 1, 1);
@@ -1098,8 +1187,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     cfg.numAttrs = 1;
     cudaLaunchKernelEx(&cfg, gemm_tc_kernel<bf16, true>, p);
   } else {
-    const int grid = tiles < num_sms() ? tiles : num_sms();
-    gemm_tc_kernel<bf16, false><<<grid, TC_THREADS, TC_SMEM, s>>>(p);
+    gemm_tc_kernel<bf16, false><<<nunits, TC_THREADS, TC_SMEM, s>>>(p);
   }
   count_launches(1);
   cudaError_t e = cudaGetLastError();

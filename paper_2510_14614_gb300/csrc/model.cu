@@ -773,11 +773,11 @@ int backward_impl(fal_handle* h) {
   Ctx c{h};
   cudaStream_t s = h->sm;
   const int BT = (int)h->BT, d = h->d;
-  // LM head: dxf = dlogits wte, dwte = dlogits^T xf (stores; the embedding adds later)
-  gemm(c, call1(BT, d, seg(h->dlogits, h->Vp, 0, Wp(h, h->wte), d, 1, h->V), epi_out(h->dU, d, OUT_F32)), s,
-       "LM head dgrad");
-  gemm(c, call1(h->V, d, seg(h->dlogits, h->Vp, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte), d, OUT_F32)), s,
-       "LM head wgrad");
+  // LM head: dwte = dlogits^T xf and dxf = dlogits wte in one launch (stores;
+  // the embedding adds later)
+  gemm(c, group_calls({call1(h->V, d, seg(h->dlogits, h->Vp, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte), d, OUT_F32)),
+                       call1(BT, d, seg(h->dlogits, h->Vp, 0, Wp(h, h->wte), d, 1, h->V), epi_out(h->dU, d, OUT_F32))}),
+       s, "LM head wgrad + dgrad");
   ln_bwd_(c, s, h->dU, nullptr, h->Xout, h->lnf_mean, h->lnf_rstd, Pp(h, h->lnf_g), nullptr, h->dX, h->dX_act,
           h->part0, Gp(h, h->lnf_g), Gp(h, h->lnf_b));
   if (h->cfg.variant != FAL_GPT) cudaMemsetAsync(h->dA1hat, 0, (size_t)BT * d * 4, s);
