@@ -777,6 +777,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       const int kind = G.kind;
       if (!mbar_wait_cluster(tfull_bar(acc), acc_phase, abort_flag)) break;
       tc_fence_after();
+      int* ord_flag = G.epi.ord_role ? G.epi.ord_flags + (long)(tile - G.tile_start) * (2 * TC_EPI_WARPS) +
+                                           (int)rank * TC_EPI_WARPS + (warp - 2)
+                                     : nullptr;
+      if (G.epi.ord_role == ORD_WAIT) {
+        // the same rows and columns of the signalling group must be in memory first
+        bool ok = true;
+        if (lane == 0) {
+          ok = flag_wait_eq(ord_flag, G.epi.ord_epoch, abort_flag);
+          fence_proxy_async_global();
+        }
+        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+          if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+          break;
+        }
+      }
       const int row0 = m0 + (int)rank * 128 + q * 32;
       const bool rd = G.epi.rd_out != nullptr;
       float rdot = 0.f;
@@ -801,6 +816,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
         else mbar_arrive_remote(map_to_rank(tempty_bar(acc), 0));
       }
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      if (G.epi.ord_role == ORD_SIGNAL) {
+        // publish this warp's 32 x 128 piece once its stores have landed
+        if (lane == 0) {
+          bulk_wait_all();
+          fence_proxy_async_global();
+          st_release_gpu(ord_flag, G.epi.ord_epoch);
+        }
+        __syncwarp();
+      }
     }
     if (lane == 0) bulk_wait_all();
     __syncwarp();
@@ -929,14 +953,10 @@ int num_sms() {
   return n;
 }
 
-// Contractions with an MN-major operand (every data- and weight-gradient GEMM)
-// run on CTA pairs, whose halved per-SM operand traffic pays off there; the
-// K-major forward GEMMs keep one CTA per 128x256 tile, which measures faster.
 int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg) {
-  bool mn = false;
-  for (int g = 0; g < c.ngroups; ++g)
-    for (int k = 0; k < c.g[g].nseg; ++k) mn = mn || c.g[g].seg[k].A.mn_major || c.g[g].seg[k].B.mn_major;
-  return gemm_tc_engine(c, mn ? TC_PAIR : TC_ONE, dev_err, s, msg);
+  // CTA pairs (256 x 256 tiles, each SM reading half of both operand tiles)
+  // are faster than single CTAs for every operand layout and shape of the model.
+  return gemm_tc_engine(c, TC_PAIR, dev_err, s, msg);
 }
 
 // How many clusters of two CTAs of `kernel` (dynamic shared memory `smem`) fit on the GPU at once.
@@ -1148,8 +1168,10 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     const EpiParams& e = c.g[g].epi;
     if (!e.ord_role) continue;
     const TcGroup& T = p.grp[g];
-    bool ok = kind == TC_ONE && T.out_tma && e.ord_flags && e.ord_role >= ORD_SIGNAL && e.ord_role <= ORD_WAIT &&
-              (long)T.m_tiles * T.n_tiles * TC_EPI_WARPS <= (long)e.ord_cap && e.rd_out == nullptr;
+    const long flags_per_tile = pair ? 2 * TC_EPI_WARPS : TC_EPI_WARPS;
+    bool ok = (kind == TC_ONE || kind == TC_PAIR) && T.out_tma && e.ord_flags && e.ord_role >= ORD_SIGNAL &&
+              e.ord_role <= ORD_WAIT && (long)T.m_tiles * T.n_tiles * flags_per_tile <= (long)e.ord_cap &&
+              e.rd_out == nullptr;
     if (ok && e.ord_role == ORD_WAIT) {
       ok = false;
       if (e.out_mode == OUT_F32_ACCUM)
@@ -1160,7 +1182,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
             ok = true;
     }
     if (!ok) {
-      if (msg) *msg = "ordered split-K needs the one-CTA engine, TMA outputs and a matching signalling group first";
+      if (msg) *msg = "ordered split-K needs the one-CTA or pair engine, TMA outputs and a matching signalling group first";
       return 1;
     }
   }

@@ -267,7 +267,7 @@ void carve(fal_handle* h, uint8_t* base) {
   h->tok = b.take<int32_t>(BT);
   h->tgt = b.take<int32_t>(BT);
   h->dev_err = b.take<int>(4);
-  h->ord_cap = (int)(((BT + 127) / 128) * (((long)d + 255) / 256) * 8);
+  h->ord_cap = (int)(((BT + 127) / 128) * (((long)d + 255) / 256) * 16);
   h->ord_flags = b.take<int>(h->ord_cap);
   h->loss = b.take<float>(4);
   h->loss_rows = b.take<float>(BT);
@@ -509,11 +509,11 @@ void up_gemm(Ctx& c, int i, cudaStream_t s) {
   gemm(c, call1((int)h->BT, h->F, seg(A.m, h->d, 0, Wp(h, p.w_up), h->d, 0, h->d), e), s, "MLP up-projection");
 }
 
-// Whether splitting an M x N output of 128 x 256 tiles in two halves of K fills
-// the last wave of the persistent grid (one CTA per SM) clearly better.
+// Whether splitting an M x N output of 256 x 256 tiles (one per pair of SMs)
+// in two halves of K fills the last wave of the persistent grid clearly better.
 bool split_k_pays(long M, long N) {
-  const long sms = num_sms(), tiles = ((M + 127) / 128) * ((N + 255) / 256);
-  auto fill = [&](long t) { return (double)t / (double)(((t + sms - 1) / sms) * sms); };
+  const long units = num_sms() / 2, tiles = ((M + 255) / 256) * ((N + 255) / 256);
+  auto fill = [&](long t) { return (double)t / (double)(((t + units - 1) / units) * units); };
   return fill(2 * tiles) > fill(tiles) + 0.05;
 }
 

@@ -137,7 +137,7 @@ def test_call_order_errors():
 
 
 # GPT-2-small width at depth 3, one sequence: the FAL residual GEMM of blocks 2
-# and 3 (24 output tiles of 128 x 256) runs as two ordered halves of K.
+# and 3 (12 output tiles of 256 x 256) runs as two ordered halves of K.
 SPLITK = synth.SHAPES["gpt2_small"].replace(layers=3, batch=1)
 
 
