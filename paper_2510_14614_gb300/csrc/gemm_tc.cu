@@ -224,6 +224,51 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep
   // the previous chunk's TMA stores must have read this buffer
   if (lane == 0) bulk_wait_read_all();
   __syncwarp();
+  if constexpr (KIND == EK_DGELU && sizeof(act_t) == 2) {
+    if (!o.out_f32 && (q.ldx & 7) == 0 && row0 + 32 <= o.M && col0 + 32 <= o.N) {
+      // Interior bf16 chunk: the pre-activation h is read with coalesced
+      // 16-byte loads (four lanes per 64-byte row segment, eight rows per
+      // load) into the upper half of the warp's buffer, in the swizzled layout
+      // of the output, from which each lane then takes its own row.
+      uint8_t* sb = reinterpret_cast<uint8_t*>(stage);
+      const act_t* aux = reinterpret_cast<const act_t*>(q.aux);
+      uint4 hv[4];
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int rr = it * 8 + (lane >> 2);
+        hv[it] = *reinterpret_cast<const uint4*>(aux + (long)(row0 + rr) * q.ldx + col0 + (lane & 3) * 8);
+      }
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int rr = it * 8 + (lane >> 2), u = lane & 3;
+        *reinterpret_cast<uint4*>(sb + 2048 + rr * 64 + ((u ^ ((rr >> 1) & 3)) << 4)) = hv[it];
+      }
+      __syncwarp();
+      const int sw = (lane >> 1) & 3;
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        const uint4 hp = *reinterpret_cast<const uint4*>(sb + 2048 + lane * 64 + ((g ^ sw) << 4));
+        const uint32_t hw[4] = {hp.x, hp.y, hp.z, hp.w};
+        uint32_t ow[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 h2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hw[j]));
+          const float a = __uint_as_float(r[8 * g + 2 * j]) * epi_gelu_grad<act_t>(h2.x);
+          const float b = __uint_as_float(r[8 * g + 2 * j + 1]) * epi_gelu_grad<act_t>(h2.y);
+          __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+          ow[j] = *reinterpret_cast<uint32_t*>(&t);
+        }
+        *reinterpret_cast<uint4*>(sb + lane * 64 + ((g ^ sw) << 4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(&p.maps[o.omap], stage_s, col0, row0);
+        bulk_commit();
+      }
+      return;
+    }
+  }
   const int row = row0 + lane;
   float4 y[8];
 #pragma unroll
@@ -287,6 +332,56 @@ __device__ __forceinline__ float rowdot_chunk(const EpiParams* ep, int M, int ro
   }
   return s;
 }
+// The same for a whole interior chunk (rows row0.., all in range): the 32 x 32
+// block of rd_src is read with coalesced 16-byte loads into the upper half of
+// the warp's buffer (swizzled like the output rows) and each lane takes its row
+// from there.  The buffer must be free of pending TMA reads.
+__device__ __forceinline__ float rowdot_chunk_staged(const EpiParams* ep, uint8_t* sb, int lane, int row0, int col0,
+                                                     const uint32_t* r) {
+  const bf16* src = reinterpret_cast<const bf16*>(ep->rd_src);
+  uint4 v[4];
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int rr = it * 8 + (lane >> 2);
+    v[it] = *reinterpret_cast<const uint4*>(src + (long)(row0 + rr) * ep->rd_ld + col0 + (lane & 3) * 8);
+  }
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int rr = it * 8 + (lane >> 2), u = lane & 3;
+    *reinterpret_cast<uint4*>(sb + 2048 + rr * 64 + ((u ^ ((rr >> 1) & 3)) << 4)) = v[it];
+  }
+  __syncwarp();
+  const int sw = (lane >> 1) & 3;
+  float s = 0.f;
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const uint4 op = *reinterpret_cast<const uint4*>(sb + 2048 + lane * 64 + ((g ^ sw) << 4));
+    const uint32_t ow[4] = {op.x, op.y, op.z, op.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 o2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
+      s += to_f(from_f<bf16>(__uint_as_float(r[8 * g + 2 * j]))) * o2.x +
+           to_f(from_f<bf16>(__uint_as_float(r[8 * g + 2 * j + 1]))) * o2.y;
+    }
+  }
+  __syncwarp();
+  return s;
+}
+
+// Row-dot share of one chunk, staged through the warp's buffer when it can be.
+template <typename act_t>
+__device__ __forceinline__ float rowdot_any(const EpiParams* ep, int M, int N, float4* stage, int lane, int row0,
+                                           int col0, const uint32_t* r) {
+  if constexpr (sizeof(act_t) == 2) {
+    if (row0 + 32 <= M && col0 + 32 <= N) {
+      if (lane == 0) bulk_wait_read_all();
+      __syncwarp();
+      return rowdot_chunk_staged(ep, reinterpret_cast<uint8_t*>(stage), lane, row0, col0, r);
+    }
+  }
+  return rowdot_chunk<act_t>(ep, M, row0 + lane, col0, r);
+}
+
 __device__ __forceinline__ void rowdot_store(const EpiParams* ep, int M, int row, int col_end, float s) {
   if (row >= M) return;
   const int T = ep->rd_T, h = (col_end - 1) / ep->rd_hd;
@@ -564,7 +659,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         TMEM_LD32(taddr, r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
         if (rd) {
-          rdot += rowdot_chunk<act_t>(&G.epi, eo.M, m0 + q * 32 + lane, col0, r);
+          rdot += rowdot_any<act_t>(&G.epi, eo.M, eo.N, stage, lane, m0 + q * 32, col0, r);
           if ((col0 + 32) % G.epi.rd_hd == 0) { rowdot_store(&G.epi, eo.M, m0 + q * 32 + lane, col0 + 32, rdot); rdot = 0.f; }
         }
         epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, m0 + q * 32, col0, r);
@@ -804,7 +899,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
         TMEM_LD32(taddr, r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
         if (rd) {
-          rdot += rowdot_chunk<act_t>(&G.epi, eo.M, row0 + lane, col0, r);
+          rdot += rowdot_any<act_t>(&G.epi, eo.M, eo.N, stage, lane, row0, col0, r);
           if ((col0 + 32) % G.epi.rd_hd == 0) { rowdot_store(&G.epi, eo.M, row0 + lane, col0 + 32, rdot); rdot = 0.f; }
         }
         epi_chunk_dispatch<act_t>(kind, p, &G.epi, ei, eo, stage, stage_s, lane, row0, col0, r);
