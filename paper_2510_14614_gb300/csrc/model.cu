@@ -67,7 +67,7 @@ struct fal_handle {
   int B = 0, T = 0, d = 0, H = 0, hd = 0, F = 0, L = 0, V = 0, Vp = 0;
   long BT = 0;
   cudaStream_t sm = nullptr, ss = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr, ev_mid = nullptr;
   std::string err;
   int state = 0;  // 0 fresh, 1 after forward, 2 after backward
   bool has_loss = false;
@@ -486,7 +486,7 @@ void join(fal_handle* h) {
 }
 
 // ------------------------------------------------------------ forward
-void qkv_and_attention(Ctx& c, int i, cudaStream_t s) {
+void qkv_and_attention(Ctx& c, int i, cudaStream_t s, cudaStream_t after_qkv = nullptr) {
   fal_handle* h = c.h;
   LayerA& A = h->la[i];
   const LayerP& p = h->lp[i];
@@ -494,6 +494,11 @@ void qkv_and_attention(Ctx& c, int i, cudaStream_t s) {
   EpiParams e = epi_out(A.qkv, 3L * d, OUT_ACT);
   e.bias = Pp(h, p.b_qkv);
   gemm(c, call1(BT, 3 * d, seg(A.u, d, 0, Wp(h, p.w_qkv), d, 0, d), e), s, "QKV projection");
+  if (after_qkv) {
+    // the other stream's work starts behind the projection, beside the attention
+    cudaEventRecord(h->ev_mid, s);
+    cudaStreamWaitEvent(after_qkv, h->ev_mid, 0);
+  }
   if (!c.ok()) return;
   h->err.clear();
   ProfScope ps(h, s, 1, attn_fwd_flops(h), "attention forward");
@@ -532,7 +537,7 @@ void layer_forward(Ctx& c, int i) {
     const bool two = h->cfg.schedule == FAL_SCHED_TWO_STREAM && h->ss != h->sm;
     if (two) {
       fork(h);
-      qkv_and_attention(c, i, h->ss);
+      qkv_and_attention(c, i, h->ss, s);
       up_gemm(c, i, s);
       join(h);
     } else {
@@ -843,7 +848,8 @@ int fal_create(const fal_config* cfg, void* workspace, size_t bytes, void* strea
   h->sm = reinterpret_cast<cudaStream_t>(stream_main);
   h->ss = stream_side ? reinterpret_cast<cudaStream_t>(stream_side) : h->sm;
   if (cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_mid, cudaEventDisableTiming) != cudaSuccess) {
     delete h;
     return FAL_ERR_CUDA;
   }
@@ -860,6 +866,7 @@ int fal_create(const fal_config* cfg, void* workspace, size_t bytes, void* strea
   if (cudaStreamSynchronize(s) != cudaSuccess) {
     cudaEventDestroy(h->ev_fork);
     cudaEventDestroy(h->ev_join);
+    if (h->ev_mid) cudaEventDestroy(h->ev_mid);
     delete h;
     return FAL_ERR_CUDA;
   }
@@ -874,6 +881,7 @@ void fal_destroy(fal_handle* h) {
   for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
   if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->ev_mid) cudaEventDestroy(h->ev_mid);
   delete h;
 }
 
