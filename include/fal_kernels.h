@@ -14,9 +14,9 @@
 extern "C" {
 #endif
 
-#define FAL_ENGINE_TCGEN05 0       /* tcgen05/TMEM GEMM fed by TMA, one CTA per 128x256 tile (used by the model) */
+#define FAL_ENGINE_TCGEN05 0       /* tcgen05/TMEM GEMM fed by TMA, one CTA per 128x256 tile */
 #define FAL_ENGINE_SIMT 1         /* plain fp32-FMA tiled GEMM */
-#define FAL_ENGINE_TCGEN05_PAIR 2  /* tcgen05/TMEM GEMM fed by TMA, CTA pairs (cta_group::2, 256x256 tiles) */
+#define FAL_ENGINE_TCGEN05_PAIR 2  /* tcgen05/TMEM GEMM fed by TMA, CTA pairs (cta_group::2, 256x256 tiles; used by the model) */
 #define FAL_ENGINE_TCGEN05_MC 3    /* tcgen05/TMEM GEMM, 128x256 tiles, clusters of two CTAs sharing B by TMA multicast */
 
 /* C[M,N] = sum_k A(m,k) B(n,k) (+ bias[n]) : the contraction of every linear map
