@@ -11,7 +11,8 @@
 //            up to the diagonal, recomputes S, dP, P and dS row-wise and
 //            accumulates dQ += dS K.
 //
-// The two passes share one kernel template.  Roles per CTA (320 threads):
+// The two passes share one body template and run in one launch (alternating
+// CTAs, heaviest blocks of both first).  Roles per CTA (320 threads):
 //   warp 0      producer: the resident 128-row tiles once (K and V, or Q and
 //               dO), then the streamed 64-row tiles through a 4-stage ring; in
 //               pass KV it also stages lse and D of each query block.
@@ -68,7 +69,7 @@ struct Bwd2Smem {
 };
 
 template <int HD, bool KV>
-__global__ void __launch_bounds__(AB2_THREADS, 1) attn_bwd2_kernel(const __grid_constant__ AttnBwd2Params p) {
+__device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) {
   using L = Bwd2Smem<HD, KV>;
   constexpr int KCH = L::KCH;
   extern __shared__ uint8_t smem_raw[];
@@ -88,7 +89,7 @@ __global__ void __launch_bounds__(AB2_THREADS, 1) attn_bwd2_kernel(const __grid_
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   // heaviest CTAs first: key block 0 (pass KV) / the last query block (pass Q)
-  const int blk = KV ? (int)blockIdx.x : p.nblk - 1 - (int)blockIdx.x;
+  const int blk = KV ? bx : p.nblk - 1 - bx;
   const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
   const int d = p.H * HD;
   const int row_base = b * p.T;
@@ -345,21 +346,30 @@ __global__ void __launch_bounds__(AB2_THREADS, 1) attn_bwd2_kernel(const __grid_
   }
 }
 
-template <int HD, bool KV>
+// Both passes in one launch (they read the same inputs and write disjoint
+// columns of dqkv): even x runs pass KV, odd x pass Q, so the heaviest blocks of
+// both go first and the two passes share one wave tail instead of two.
+template <int HD>
+__global__ void __launch_bounds__(AB2_THREADS, 1) attn_bwd2_kernel(const __grid_constant__ AttnBwd2Params p) {
+  if (blockIdx.x & 1) attn_bwd2_body<HD, false>(p, (int)(blockIdx.x >> 1));
+  else attn_bwd2_body<HD, true>(p, (int)(blockIdx.x >> 1));
+}
+
+template <int HD>
 int launch_bwd2(const AttnBwd2Params& p, int BH, cudaStream_t s, std::string* msg) {
-  using L = Bwd2Smem<HD, KV>;
-  static_assert(L::TOTAL <= 232448, "attention backward shared memory");
+  constexpr int smem = Bwd2Smem<HD, true>::TOTAL > Bwd2Smem<HD, false>::TOTAL ? Bwd2Smem<HD, true>::TOTAL
+                                                                               : Bwd2Smem<HD, false>::TOTAL;
+  static_assert(smem <= 232448, "attention backward shared memory");
   static bool set = false;
   if (!set) {
-    if (cudaFuncSetAttribute(attn_bwd2_kernel<HD, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
-        cudaSuccess) {
+    if (cudaFuncSetAttribute(attn_bwd2_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) {
       if (msg) *msg = "attention backward smem attribute failed";
       return 4;
     }
     set = true;
   }
-  dim3 grid(p.nblk, BH);
-  attn_bwd2_kernel<HD, KV><<<grid, AB2_THREADS, L::TOTAL, s>>>(p);
+  dim3 grid(2 * p.nblk, BH);
+  attn_bwd2_kernel<HD><<<grid, AB2_THREADS, smem, s>>>(p);
   count_launches(1);
   return 0;
 }
@@ -389,13 +399,8 @@ int attn_bwd2_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx,
   p.scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
   p.err = dev_err;
   int r;
-  if (hd == 64) {
-    r = launch_bwd2<64, true>(p, B * H, s, msg);
-    if (!r) r = launch_bwd2<64, false>(p, B * H, s, msg);
-  } else {
-    r = launch_bwd2<128, true>(p, B * H, s, msg);
-    if (!r) r = launch_bwd2<128, false>(p, B * H, s, msg);
-  }
+  if (hd == 64) r = launch_bwd2<64>(p, B * H, s, msg);
+  else r = launch_bwd2<128>(p, B * H, s, msg);
   if (r) return r;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) { if (msg) *msg = std::string("attention backward launch: ") + cudaGetErrorString(e); return 4; }
