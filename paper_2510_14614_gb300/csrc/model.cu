@@ -676,8 +676,14 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   const LayerP& p = h->lp[i];
   const int BT = (int)h->BT, d = h->d;
   if (!skip_wo) {
+    // dctx also yields the attention backward's D = rowsum(dctx * ctx) per head
+    EpiParams edc = epi_out(h->dctx, d, OUT_ACT);
+    if (h->bf) {
+      edc.rd_src = A.ctx; edc.rd_ld = d; edc.rd_out = h->dvec; edc.rd_hd = h->hd; edc.rd_T = h->T; edc.rd_H = h->H;
+      d_ready = true;
+    }
     gemm(c, group_calls({call1(d, d, wgrad_seg(h, da_act, d, A.ctx, d), wgrad_out(h, p.w_o, d)),
-                         call1(BT, d, dgrad_seg(h, da_act, d, p.w_o, d), epi_out(h->dctx, d, OUT_ACT))}),
+                         call1(BT, d, dgrad_seg(h, da_act, d, p.w_o, d), edc)}),
          s, "attention out wgrad + dgrad");
     colsum_(c, s, part, da, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o), nullptr, 0);
   }
