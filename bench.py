@@ -345,7 +345,7 @@ def main():
         "model_tflops": mfu,
         "frac_of_peak": {"burst": mfu / peak_burst, "sustained": mfu / peak_sus, "peak_kind": peak_kind},
         "roofline": {
-            "kernel": "gemm_tc_kernel (tcgen05 GEMM, all launches of the timed steps)",
+            "kernel": "gemm_tc2_kernel (tcgen05 GEMM on CTA pairs, all launches of the timed steps)",
             "bound": "tensor", "achieved": gemm_tflops, "peak": peak_sus, "unit": "TFLOP/s",
             "frac": (gemm_tflops / peak_sus) if gemm_tflops else None,
             "traffic": gemm_traffic(args.workload if args.layers is None and args.batch is None else "",
