@@ -65,6 +65,22 @@ def dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(x, world, torch):
+    """The slowest rank's time: replicas run independent steps, the job takes
+    as long as its slowest member (max all-reduce; identity on one rank)."""
+    if world <= 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, n, seconds):
+    """Whole-job tokens/s of n replicas that each processed tokens_per_rank in
+    `seconds` (the max over ranks): weak scaling, no data-path exchange."""
+    return tokens_per_rank * n / seconds
+
+
 def workload_config(s, variant, schedule, n):
     return {
         "workload": f"{s.name} {variant.upper() if variant != 'falplus' else 'FAL+'}: L={s.layers} d_model={s.d_model} "
@@ -266,11 +282,8 @@ def time_variant(args, s, variant, schedule, torch, fal, dev, n, world, rank, pe
     launches = fal.launch_count() - n0
     m.profile_enable(False)
     prof = m.profile_read()
-    ms = ev0.elapsed_time(ev1) / args.steps
+    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, world, torch)
     if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
         torch.distributed.barrier()
     loss1 = m.loss()
     res = {"ms": ms, "launches": launches / args.steps * args.steps, "prof": prof, "clocks": clk.summary(),
@@ -286,11 +299,7 @@ def time_variant(args, s, variant, schedule, torch, fal, dev, n, world, rank, pe
         t0 = time.perf_counter()
         for _ in range(args.steps):
             m.train_step(tok_h, tgt_h, sync=True)
-        e2e_s = (time.perf_counter() - t0) / args.steps
-        if world > 1:
-            t = torch.tensor([e2e_s], dtype=torch.float64)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_s = float(t.item())
+        e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, world, torch)
         res["e2e_s"] = e2e_s
         res["h2d"] = tok_h.numel() * 4 * 2
         res["d2h"] = 4
@@ -329,7 +338,7 @@ def main():
 
     tokens = s.tokens * n
     ms = main_res["ms"]
-    value = tokens / (ms / 1e3)
+    value = job_throughput(s.tokens, n, ms / 1e3)
     flops = synth.model_flops_per_step(s)
     peak_burst = peaks.get("bf16_tflops", 1900.0)
     peak_sus = peaks.get("bf16_tflops_sustained", 1700.0)
