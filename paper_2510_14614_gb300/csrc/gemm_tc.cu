@@ -200,6 +200,11 @@ template <typename act_t, int KIND>
 __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep, const EpiIn q, const EpiOut o,
                                           float4* stage, uint32_t stage_s, int lane, int row0, int col0,
                                           const uint32_t* r) {
+  // Every path below writes this buffer: the TMA stores of earlier chunks must
+  // have read it (a weight-gradient tile with the AdamW epilogue may follow a
+  // data-gradient tile in the same warp when the data gradient is the deeper one).
+  if (lane == 0) bulk_wait_read_all();
+  __syncwarp();
   if constexpr (KIND == EK_ADAMW) {
     epi_adamw_chunk(ep, o.M, o.N, stage, lane, row0, col0, r);
     return;
@@ -221,9 +226,6 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep
     __syncwarp();
     return;
   }
-  // the previous chunk's TMA stores must have read this buffer
-  if (lane == 0) bulk_wait_read_all();
-  __syncwarp();
   if constexpr (KIND == EK_DGELU && sizeof(act_t) == 2) {
     if (!o.out_f32 && (q.ldx & 7) == 0 && row0 + 32 <= o.M && col0 + 32 <= o.N) {
       // Interior bf16 chunk: the pre-activation h is read with coalesced
