@@ -36,7 +36,8 @@ extern "C" {
 #define FAL_OK 0
 #define FAL_ERR_ARG 1         /* null pointer, bad shape, bad alignment, token id out of range */
 #define FAL_ERR_STATE 2       /* call order (e.g. backward without a forward) */
-#define FAL_ERR_WORKSPACE 3   /* workspace smaller than fal_workspace_size() */
+#define FAL_ERR_WORKSPACE 3   /* workspace smaller than fal_workspace_size(), or a problem larger than the
+                                 fixed scratch of fal_kernel_attention_bwd_noalloc (fal_kernels.h) */
 #define FAL_ERR_CUDA 4        /* a CUDA runtime/driver call failed */
 #define FAL_ERR_TIMEOUT 5     /* a bounded device-side wait expired (kernel returned early) */
 #define FAL_ERR_UNSUPPORTED 6 /* configuration valid but not implemented on this path */

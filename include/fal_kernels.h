@@ -17,7 +17,6 @@ extern "C" {
 #define FAL_ENGINE_TCGEN05 0       /* tcgen05/TMEM GEMM fed by TMA, one CTA per 128x256 tile */
 #define FAL_ENGINE_SIMT 1         /* plain fp32-FMA tiled GEMM */
 #define FAL_ENGINE_TCGEN05_PAIR 2  /* tcgen05/TMEM GEMM fed by TMA, CTA pairs (cta_group::2, 256x256 tiles; used by the model) */
-#define FAL_ENGINE_TCGEN05_MC 3    /* tcgen05/TMEM GEMM, 128x256 tiles, clusters of two CTAs sharing B by TMA multicast */
 
 /* C[M,N] = sum_k A(m,k) B(n,k) (+ bias[n]) : the contraction of every linear map
  * of the blocks (Eq. 1, Eq. 2) and of their gradients.
@@ -60,12 +59,15 @@ int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const
  * holds it until the process exits.  The call needs
  * B*H*T <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS and returns
  * FAL_ERR_WORKSPACE (launching nothing) above that.  It never calls cudaMalloc,
- * cudaFree or any allocating routine.  The first call on each device looks up
- * the array's device address (cudaGetSymbolAddress, with that device current);
- * make that first call before any stream capture.  All calls share the one
- * array and each call rewrites what it reads, so calls that overlap on the GPU
- * (different streams, or several host threads on one device) race: serialize
- * them. */
+ * cudaFree or any allocating routine.  Every call made while `stream` is not
+ * being captured looks up the array's device address in the current device's
+ * context (cudaGetSymbolAddress), so the address stays right after a device
+ * reset; a call made while `stream` is being captured uses the address found
+ * by an earlier call on the same device and context, and returns
+ * FAL_ERR_STATE if there was none: make one call before any stream capture.
+ * All calls share the one array and each call rewrites what it reads, so calls
+ * that overlap on the GPU (different streams, or several host threads on one
+ * device) race: serialize them. */
 #define FAL_NOALLOC_ATTN_SCRATCH_FLOATS (4u * 1024u * 1024u)
 int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
                                      const void* dctx, void* dqkv, void* stream);

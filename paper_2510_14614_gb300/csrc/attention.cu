@@ -1,9 +1,11 @@
 // Causal multi-head attention, forward and backward (the MHA_i of every block).
 //
-// bf16 path: the tcgen05 kernels live in attention_tc.cu; this file holds the
-// backward's pre-pass (D = rowsum(dO * O), zeroed dQ accumulator) and post-pass
-// (dQ accumulator -> bf16), the fp32 debug kernels (one thread per query row,
-// plain fp32 arithmetic) and the allocation-free backward entry point.
+// bf16 path: the tcgen05 kernels live in attention_tc.cu (forward) and
+// attention_bwd_tc.cu (backward); this file holds the backward's pre-pass
+// D = rowsum(dO * O) for the kernel-level entry points (the model takes D from
+// the epilogue of the GEMM that produces dO), the fp32 debug kernels (one thread
+// per query row, plain fp32 arithmetic) and the allocation-free backward entry
+// point.
 //
 // Scores: S = Q K^T / sqrt(hd), key j visible to query t iff j <= t.  The
 // saved log-sum-exp is in log2 units of S*log2(e).
@@ -17,25 +19,25 @@ namespace {
 constexpr float LOG2E = 1.4426950408889634f;
 
 // ------------------------------------------------------------ backward (bf16)
-// D[b,h,t] = sum_c dO[t,c] * O[t,c].
+// D[b,h,t] = sum_c dO[t,c] * O[t,c]: one warp per (token row, head), in a
+// grid-stride loop over all B*T*H of them (any B*T, no grid-dimension limit).
 __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx,
-                                    float* __restrict__ dvec, int T, int H, int hd) {
-  const int warps = blockDim.x / 32;
-  const int w = blockIdx.x * warps + threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int d = H * hd;
-  const long rows = (long)gridDim.y;  // unused guard
-  (void)rows;
-  const int bt = blockIdx.y;           // token row
-  if (w >= H) return;
-  const int h = w;
-  const bf16* o = ctx + (long)bt * d + h * hd;
-  const bf16* g = dctx + (long)bt * d + h * hd;
-  float acc = 0.f;
-  for (int c = lane; c < hd; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(g[c]);
-  acc = warp_sum(acc);
-  if (lane == 0) {
-    const int b = bt / T, t = bt % T;
-    dvec[((long)b * H + h) * T + t] = acc;
+                                    float* __restrict__ dvec, long rows, int T, int H, int hd) {
+  const int lane = threadIdx.x % 32;
+  const long nwarps = (long)gridDim.x * (blockDim.x / 32);
+  const long d = (long)H * hd;
+  for (long w = blockIdx.x * (long)(blockDim.x / 32) + threadIdx.x / 32; w < rows * H; w += nwarps) {
+    const long bt = w / H;
+    const int h = (int)(w - bt * H);
+    const bf16* o = ctx + bt * d + (long)h * hd;
+    const bf16* g = dctx + bt * d + (long)h * hd;
+    float acc = 0.f;
+    for (int c = lane; c < hd; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(g[c]);
+    acc = warp_sum(acc);
+    if (lane == 0) {
+      const long b = bt / T, t = bt % T;
+      dvec[(b * H + h) * T + t] = acc;
+    }
   }
 }
 
@@ -148,11 +150,12 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
   const int d = H * hd;
   if (act_bf16) {
     if (hd != 64 && hd != 128) { if (msg) *msg = "bf16 attention needs head_dim 64 or 128"; return 6; }
-    const int wpb = 4;
-    dim3 pg((H + wpb - 1) / wpb, (unsigned)rows);
     if (!d_ready) {
-      attn_bwd_pre_kernel<<<pg, wpb * 32, 0, s>>>(reinterpret_cast<const bf16*>(ctx),
-                                                 reinterpret_cast<const bf16*>(dctx), dvec, T, H, hd);
+      const int wpb = 8;
+      const long warps = rows * H;
+      const long want = (warps + wpb - 1) / wpb, cap = 16L * num_sms();
+      attn_bwd_pre_kernel<<<(unsigned)(want < cap ? want : cap), wpb * 32, 0, s>>>(
+          reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx), dvec, rows, T, H, hd);
       count_launches(1);
     }
     const int r = attn_bwd2_tc(B, T, H, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
@@ -174,9 +177,10 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
 
 // ------------------------------------------------------------ allocation-free entry point
 // Scratch for fal_kernel_attention_bwd_noalloc: a fixed file-scope device array
-// (dQ accumulator followed by the D = rowsum(dO * O) vector).  Host code only
+// that receives the D = rowsum(dO * O) vector, [B, H, T] fp32.  Host code only
 // ever sees a stand-in for this symbol, so its device address is looked up
-// once per device with cudaGetSymbolAddress while that device is current.
+// with cudaGetSymbolAddress while the caller's device is current.
+#include <cuda.h>
 #include <mutex>
 
 #include "../../include/fal.h"
@@ -189,19 +193,52 @@ static __device__ __align__(256) float g_noalloc_attn_scratch[kNoAllocFloats];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
+// Address of the array per device, and the CUDA context it was looked up in:
+// after a device reset (or under another context) the module is loaded anew
+// and the array may sit elsewhere.
 float* g_noalloc_ptr[kMaxDevices] = {};
+CUcontext g_noalloc_ctx[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device (looked up once).
-int noalloc_scratch(float** out) {
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  });
+  return fn;
+}
+
+// Device address of the scratch array in the current context.  Outside stream
+// capture the address is looked up on every call (cheap once the module is
+// loaded), so a cached value never outlives a device reset; while `s` is being
+// captured no runtime lookup is made and the address cached for this device
+// and context by an earlier call is used.
+int noalloc_scratch(cudaStream_t s, float** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FAL_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return FAL_ERR_UNSUPPORTED;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cap) != cudaSuccess) return FAL_ERR_CUDA;
+  // The runtime makes the device's primary context current on first use; the
+  // call above has done that, so the driver now reports the context in use.
+  CUcontext ctx = nullptr;
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get || get(&ctx) != CUDA_SUCCESS) return FAL_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_attn_scratch) != cudaSuccess || !p) return FAL_ERR_CUDA;
-    g_noalloc_ptr[dev] = static_cast<float*>(p);
+  if (cap != cudaStreamCaptureStatusNone) {
+    if (!g_noalloc_ptr[dev] || g_noalloc_ctx[dev] != ctx) return FAL_ERR_STATE;
+    *out = g_noalloc_ptr[dev];
+    return FAL_OK;
   }
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_attn_scratch) != cudaSuccess || !p) return FAL_ERR_CUDA;
+  g_noalloc_ptr[dev] = static_cast<float*>(p);
+  g_noalloc_ctx[dev] = ctx;
   *out = g_noalloc_ptr[dev];
   return FAL_OK;
 }
@@ -214,7 +251,7 @@ extern "C" int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, con
   const size_t need = (size_t)B * H * T;
   if (need > kNoAllocFloats) return FAL_ERR_WORKSPACE;
   float* scratch = nullptr;
-  const int rc = noalloc_scratch(&scratch);
+  const int rc = noalloc_scratch(reinterpret_cast<cudaStream_t>(stream), &scratch);
   if (rc != FAL_OK) return rc;
   std::string msg;
   // attn_bwd's first kernel writes every D entry before it is read, so nothing

@@ -438,25 +438,16 @@ __device__ __forceinline__ int group_of(const TcParams& p, int tile) {
   return g;
 }
 
-// MC: a cluster of two CTAs owns a 256-row band of output tiles; CTA `rank`
-// computes rows m0 + 128 * rank.
-template <bool MC>
-__device__ __forceinline__ void decode_tile(const TcParams& p, int tile, uint32_t rank, int& g, int& m0, int& n0) {
+__device__ __forceinline__ void decode_tile(const TcParams& p, int tile, int& g, int& m0, int& n0) {
   g = group_of(p, tile);
   const TcGroup& G = p.grp[g];
   int mt, nt;
   tile_mn(G, tile - G.tile_start, mt, nt);
-  m0 = mt * (MC ? 2 * TC_BM : TC_BM) + (int)rank * TC_BM;
+  m0 = mt * TC_BM;
   n0 = nt * TC_BN;
 }
 
-// MC = true: launched in clusters of two CTAs on vertically adjacent tiles that
-// share their B tile.  Each CTA loads its own A tile and one half of the B
-// tile, multicast into both CTAs' shared memory, so the L2-to-SM traffic per
-// CTA drops from 48 KB to 32 KB per 64-deep K step.  A stage may be refilled
-// only when both CTAs' MMAs have read it: every MMA commit arrives on the
-// empty barrier of both CTAs (count 2).
-template <typename act_t, bool MC>
+template <typename act_t>
 __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -473,11 +464,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(bar_ptr + 8 * (2 * TC_STAGES + 5) + 4);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const uint32_t rank = MC ? cluster_ctarank() : 0u;
-  const int unit = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;     // this CTA's (or cluster's) tile stream
-  const int nunits = MC ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  const int unit = (int)blockIdx.x, nunits = (int)gridDim.x;  // this CTA's tile stream
   if (threadIdx.x == 0) {
-    for (int s = 0; s < TC_STAGES; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), MC ? 2 : 1); }
+    for (int s = 0; s < TC_STAGES; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
     for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), TC_EPI_WARPS); }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -490,13 +479,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  if (MC) cluster_sync_all(); else __syncthreads();
+  __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // On a timeout the peer CTA is told to stop too (it may be feeding this CTA).
-  auto abort_peer = [&]() {
-    if (MC) st_cluster_u32(map_to_rank(smem_u32(const_cast<uint32_t*>(abort_flag)), rank ^ 1u), 1u);
-  };
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
@@ -506,14 +491,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     bool ok = true;
     for (int ti = 0, tile; ok && (tile = tile_at(p, unit, nunits, ti)) >= 0; ++ti) {
       int g, m0, n0;
-      decode_tile<MC>(p, tile, rank, g, m0, n0);
+      decode_tile(p, tile, g, m0, n0);
       const TcGroup& G = p.grp[g];
       for (int s = 0; s < G.nseg && ok; ++s) {
         const CUtensorMap* am = &p.maps[G.amap[s]];
         const CUtensorMap* bm = &p.maps[G.bmap[s]];
         for (int kb = 0; kb < G.kb[s]; ++kb) {
-          if (!(MC ? mbar_wait_cluster(empty_bar(stage), phase ^ 1u, abort_flag)
-                   : mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag))) { ok = false; break; }
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag)) { ok = false; break; }
           if (lane == 0) {
             const uint32_t fb = full_bar(stage);
             const uint32_t sa = base + stage * TC_STAGE_BYTES;
@@ -526,16 +510,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
             } else {
               tma_load_2d(sa, am, k0, m0, fb);
             }
-            if (MC) {
-              // this CTA's half of the shared B tile, delivered to both CTAs
-              if (G.b_mn) {
-#pragma unroll
-                for (int j = 2 * (int)rank; j < 2 * (int)rank + 2; ++j)
-                  tma_load_2d_mc(sb + j * TC_MN_CHUNK_BYTES, bm, n0 + 64 * j, k0, fb, 0x3);
-              } else {
-                tma_load_2d_mc(sb + rank * (TC_B_BYTES / 2), bm, k0, n0 + (int)rank * (TC_BN / 2), fb, 0x3);
-              }
-            } else if (G.b_mn) {
+            if (G.b_mn) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) tma_load_2d(sb + j * TC_MN_CHUNK_BYTES, bm, n0 + 64 * j, k0, fb);
             } else {
@@ -549,16 +524,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         }
       }
     }
-    if (MC && ok) {
-      // Every stage must have been released by both CTAs' MMAs before this
-      // CTA may leave: the peer's commits arrive on these barriers.
-      for (int i = 0; i < TC_STAGES && ok; ++i) {
-        if (!mbar_wait_cluster(empty_bar(stage), phase ^ 1u, abort_flag)) ok = false;
-        if (++stage == TC_STAGES) { stage = 0; phase ^= 1u; }
-      }
-    }
     if (!ok) {
-      if (lane == 0) abort_peer();
       // Let every copy this CTA issued land before shared memory is released.
       for (int s = 0; s < TC_STAGES; ++s) {
         if (!(issued_mask & (1u << s))) continue;
@@ -603,7 +569,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
             tc_mma(d_tmem, adesc + so + k * astep, bdesc + so + k * bstep, idesc, accum);
             accum = 1;
           }
-          if (MC) tc_commit_mc(empty_bar(stage), 0x3); else tc_commit(empty_bar(stage));
+          tc_commit(empty_bar(stage));
           issued_any = true;
           if (++stage == TC_STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -611,7 +577,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         tc_commit(tfull_bar(acc));
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
-      if (!ok) abort_peer();
       if (!ok && issued_any) {
         // Wait for this thread's MMAs to finish before TMEM is freed.
         tc_commit(drain_bar);
@@ -630,7 +595,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     uint32_t acc_phase = 0;
     for (int ti = 0, tile; (tile = tile_at(p, unit, nunits, ti)) >= 0; ++ti) {
       int g, m0, n0;
-      decode_tile<MC>(p, tile, rank, g, m0, n0);
+      decode_tile(p, tile, g, m0, n0);
       const TcGroup& G = p.grp[g];
       const EpiOut eo = epi_out_of(G);
       const EpiIn ei = epi_in(G.epi);
@@ -685,7 +650,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   }
 
   tc_fence_before();
-  if (MC) cluster_sync_all(); else __syncthreads();
+  __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
@@ -1145,22 +1110,19 @@ const int* tile_schedule(const GemmCall& c, const TcParams& p, int nunits) {
 int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, std::string* msg) {
   if (!get_encoder(msg)) return 4;
   static bool attr_set = false;
-  static int pair_clusters = 0, mc_clusters = 0;
+  static int pair_clusters = 0;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<bf16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(gemm_tc_kernel<bf16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(gemm_tc2_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, T2_SMEM);
     if (e != cudaSuccess) { if (msg) *msg = std::string("gemm_tc smem attribute: ") + cudaGetErrorString(e); return 4; }
     pair_clusters = max_pair_clusters(gemm_tc2_kernel<bf16>, T2_SMEM);
-    mc_clusters = max_pair_clusters(gemm_tc_kernel<bf16, true>, TC_SMEM);
     attr_set = true;
   }
-  if (kind < TC_ONE || kind > TC_MULTICAST) { if (msg) *msg = "unknown tcgen05 GEMM kind"; return 1; }
-  const bool pair = kind == TC_PAIR, mc = kind == TC_MULTICAST;
-  const int bm = pair ? T2_TILE : (mc ? 2 * TC_BM : TC_BM), bn = pair ? T2_TILE : TC_BN;
-  const int a_rows = 128, b_rows = (pair || mc) ? 128 : TC_BN;  // K-major TMA box heights per CTA
+  if (kind != TC_ONE && kind != TC_PAIR) { if (msg) *msg = "unknown tcgen05 GEMM kind"; return 1; }
+  const bool pair = kind == TC_PAIR;
+  const int bm = pair ? T2_TILE : TC_BM, bn = pair ? T2_TILE : TC_BN;
+  const int a_rows = 128, b_rows = pair ? 128 : TC_BN;  // K-major TMA box heights per CTA
   TcParams p;
   memset(&p, 0, sizeof(p));
   int nmaps = 0, tiles = 0;
@@ -1176,7 +1138,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     {
       // Bands of about one wave of tiles when a column of tiles is narrower
       // than the machine: the A rows of a band are then read from DRAM once.
-      const int conc = pair ? pair_clusters : (mc ? mc_clusters : num_sms());
+      const int conc = pair ? pair_clusters : num_sms();
       T.band_m = (T.n_tiles <= conc) ? (conc / T.n_tiles > 1 ? conc / T.n_tiles : 1) : 0;
     }
     T.epi = G.epi;
@@ -1266,7 +1228,7 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     if (!e.ord_role) continue;
     const TcGroup& T = p.grp[g];
     const long flags_per_tile = pair ? 2 * TC_EPI_WARPS : TC_EPI_WARPS;
-    bool ok = (kind == TC_ONE || kind == TC_PAIR) && T.out_tma && e.ord_flags && e.ord_role >= ORD_SIGNAL &&
+    bool ok = T.out_tma && e.ord_flags && e.ord_role >= ORD_SIGNAL &&
               e.ord_role <= ORD_WAIT && (long)T.m_tiles * T.n_tiles * flags_per_tile <= (long)e.ord_cap &&
               e.rd_out == nullptr;
     if (ok && e.ord_role == ORD_WAIT) {
@@ -1286,27 +1248,14 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
   p.total_tiles = tiles;
   p.err = dev_err;
   if (tiles == 0) return 0;
-  const int cap = pair ? pair_clusters : (mc ? mc_clusters : num_sms());
+  const int cap = pair ? pair_clusters : num_sms();
   const int nunits = tiles < cap ? tiles : cap;
   p.sched = tile_schedule(c, p, nunits);
   if (pair) {
     const int clusters = nunits;
     gemm_tc2_kernel<bf16><<<2 * clusters, TC_THREADS, T2_SMEM, s>>>(p);
-  } else if (mc) {
-    const int clusters = nunits;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * clusters, 1, 1);
-    cfg.blockDim = dim3(TC_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = TC_SMEM;
-    cfg.stream = s;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = 2; attr.val.clusterDim.y = 1; attr.val.clusterDim.z = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, gemm_tc_kernel<bf16, true>, p);
   } else {
-    gemm_tc_kernel<bf16, false><<<nunits, TC_THREADS, TC_SMEM, s>>>(p);
+    gemm_tc_kernel<bf16><<<nunits, TC_THREADS, TC_SMEM, s>>>(p);
   }
   count_launches(1);
   cudaError_t e = cudaGetLastError();

@@ -65,9 +65,8 @@ int gemm_simt(const GemmCall& c, int in_bf16, int act_bf16, cudaStream_t s, std:
 // tcgen05/TMEM GEMM fed by TMA (bf16 operands, fp32 accumulation, bf16 activations).
 int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg);
 // TC_ONE: one CTA per 128x256 tile; TC_PAIR: CTA pairs (cta_group::2, 256x256
-// tiles); TC_MULTICAST: one CTA per 128x256 tile, clusters of two sharing the
-// B tile through TMA multicast.
-enum TcKind { TC_ONE = 0, TC_PAIR = 1, TC_MULTICAST = 2 };
+// tiles).
+enum TcKind { TC_ONE = 0, TC_PAIR = 1 };
 int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, std::string* msg);
 
 // ---------------------------------------------------------------- attention

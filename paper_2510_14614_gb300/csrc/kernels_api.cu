@@ -17,8 +17,7 @@ int fal_kernel_gemm(int M, int N, int K, const void* A, long lda, int a_mn_major
                     int b_mn_major, int in_f32, const float* bias, void* C, long ldc, int c_f32, int engine,
                     int* dev_err, void* stream) {
   if (M < 0 || N < 0 || K <= 0 || !A || !B || !C) return FAL_ERR_ARG;
-  if (engine != FAL_ENGINE_TCGEN05 && engine != FAL_ENGINE_SIMT && engine != FAL_ENGINE_TCGEN05_PAIR &&
-      engine != FAL_ENGINE_TCGEN05_MC)
+  if (engine != FAL_ENGINE_TCGEN05 && engine != FAL_ENGINE_SIMT && engine != FAL_ENGINE_TCGEN05_PAIR)
     return FAL_ERR_ARG;
   if (engine != FAL_ENGINE_SIMT && in_f32) return FAL_ERR_ARG;
   if (ldc < N || lda < (a_mn_major ? M : K) || ldb < (b_mn_major ? N : K)) return FAL_ERR_ARG;
@@ -35,10 +34,7 @@ int fal_kernel_gemm(int M, int N, int K, const void* A, long lda, int a_mn_major
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   std::string msg;
   int r = engine == FAL_ENGINE_SIMT ? gemm_simt(c, in_f32 ? 0 : 1, 1, s, &msg)
-                                    : gemm_tc_engine(c,
-                                                     engine == FAL_ENGINE_TCGEN05_PAIR ? TC_PAIR
-                                                     : engine == FAL_ENGINE_TCGEN05_MC ? TC_MULTICAST
-                                                                                       : TC_ONE,
+                                    : gemm_tc_engine(c, engine == FAL_ENGINE_TCGEN05_PAIR ? TC_PAIR : TC_ONE,
                                                      dev_err, s, &msg);
   return map_rc(r);
 }

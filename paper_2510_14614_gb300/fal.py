@@ -19,7 +19,7 @@ FAL_OK, FAL_ERR_ARG, FAL_ERR_STATE, FAL_ERR_WORKSPACE, FAL_ERR_CUDA, FAL_ERR_TIM
 VARIANT = {"gpt": 0, "fal": 1, "falplus": 2}
 PRECISION = {"bf16": 0, "fp32": 1}
 SCHEDULE = {"serial": 0, "two_stream": 1}
-ENGINE = {"tcgen05": 0, "simt": 1, "tcgen05_pair": 2, "tcgen05_mc": 3}
+ENGINE = {"tcgen05": 0, "simt": 1, "tcgen05_pair": 2}
 
 
 class FalConfig(ctypes.Structure):

@@ -41,7 +41,7 @@ def _noalloc(qkv, ctx, lse, dctx, B, T, H, hd):
     return code, dqkv
 
 
-@pytest.mark.parametrize("B,T,H,hd", [(2, 200, 2, 64), (1, 130, 2, 128)])
+@pytest.mark.parametrize("B,T,H,hd", [(2, 200, 2, 64), (1, 130, 2, 128), (520, 128, 1, 64)])
 def test_noalloc_matches_allocating_entry_point_twice(B, T, H, hd):
     import torch
     from paper_2510_14614_gb300 import fal
