@@ -1,12 +1,28 @@
 #!/usr/bin/env python
-"""Training throughput (tokens/s: forward + backward + AdamW) of a FAL decoder
-stack on GB300 through libfal's C ABI, with the same library's sequential GPT
-baseline, the GEMM roofline fraction, and the fp64 oracle on the host cores.
+"""Training throughput (tokens/s: forward + backward + AdamW) of FAL / FAL+
+decoder stacks on GB300 through libfal's C ABI, beside the same library's
+sequential GPT baseline, with the fraction of the dense BF16 peak, the GEMM
+roofline, and the fp64 oracle timed on the host cores.
 
-Default workload: the 1.3B-shaped FAL stack (24 layers, d_model 2048, 16 heads
-of 128, d_ff 8192, seq 2048, batch 4, vocab 50257), bf16 with fp32
-accumulation, seeded synthetic tokens.  Every step reads > 2.6 GB of bf16
-weights plus activations, far above the 129 MB L2, so no flush is needed.
+Headline workload: the 1.3B-shaped FAL stack (24 layers, d_model 2048, 16 heads
+of 128, d_ff 8192, seq 2048, batch 4, vocab 50257), two-stream schedule, bf16
+operands with fp32 accumulation, seeded synthetic tokens.  Every step reads
+> 2.6 GB of bf16 weights plus activations, far above the 129 MB L2, so no
+flush is needed between steps.
+
+One JSON line carries, besides the headline (timed with profiling off):
+  e2e           the same step through fal_train_step with host token buffers
+                and the loss read back every step;
+  roofline      the tcgen05 GEMMs' algorithmic FLOPs over their CUDA-event time
+                in a separate profiled pass;
+  fal_serial    the same FAL stack with both branches on one stream (isolates
+                the branch concurrency of Sec. 4.2 from the fused residual GEMM);
+  gpt_baseline  the same library's sequential GPT stack on the same shape;
+  configs       the other benchmark shapes (GPT-2 small / medium / XL): FAL or
+                FAL+ beside GPT, tokens/s and fraction of peak;
+  attention_isolated  forward and backward attention kernels timed alone on one
+                layer of the headline shape;
+  cpu_baseline  a measured sample of one fp64 oracle training step (OracleSample).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--workload gpt_1p3b|gpt2_small|gpt2_medium|gpt2_xl] [--variant fal|falplus|gpt]
@@ -31,9 +47,14 @@ from paper_2510_14614_gb300 import synth  # noqa: E402
 
 METRIC = "train tokens/s on 1 GB300 (FAL vs own GPT baseline); % of dense BF16 peak"
 UNIT = "tokens/s"
+# The other benchmark shapes and the variants each is reported with.
+CONFIG_ARMS = (("gpt2_small", ("fal", "gpt")), ("gpt2_medium", ("falplus", "gpt")),
+               ("gpt2_xl", ("fal", "falplus", "gpt")))
+REF_SEQ = 128          # tokens per timed step of the reference (oracle) arm
+CPU_SEQ = 512          # tokens of the oracle step timed for cpu_baseline
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
@@ -42,11 +63,13 @@ def parse():
     ap.add_argument("--workload", default="gpt_1p3b", choices=[k for k in synth.SHAPES if k != "tiny"])
     ap.add_argument("--variant", default="fal", choices=list(synth.VARIANTS))
     ap.add_argument("--schedule", default="two_stream", choices=["serial", "two_stream"])
-    ap.add_argument("--no-baseline", action="store_true", help="skip the same-library GPT baseline")
+    ap.add_argument("--no-baseline", action="store_true", help="skip the GPT and FAL-serial arms of the headline shape")
+    ap.add_argument("--no-configs", action="store_true", help="skip the other benchmark shapes")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--arm-steps", type=int, default=5, help="timed steps of each extra arm")
     ap.add_argument("--layers", type=int, default=None, help="override depth (small profiling cases only)")
     ap.add_argument("--batch", type=int, default=None, help="override batch (small profiling cases only)")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def shape_of(args):
@@ -81,10 +104,14 @@ def job_throughput(tokens_per_rank, n, seconds):
     return tokens_per_rank * n / seconds
 
 
+def variant_name(v):
+    return {"fal": "FAL", "falplus": "FAL+", "gpt": "GPT"}[v]
+
+
 def workload_config(s, variant, schedule, n):
     return {
-        "workload": f"{s.name} {variant.upper() if variant != 'falplus' else 'FAL+'}: L={s.layers} d_model={s.d_model} "
-                    f"heads={s.heads} (head_dim {s.head_dim}) d_ff={s.d_ff} seq={s.seq} batch={s.batch} vocab={s.vocab}",
+        "workload": f"{s.name} {variant_name(variant)}: L={s.layers} d_model={s.d_model} heads={s.heads} "
+                    f"(head_dim {s.head_dim}) d_ff={s.d_ff} seq={s.seq} batch={s.batch} vocab={s.vocab}",
         "variant": variant,
         "schedule": schedule,
         "global_batch": s.batch * n,
@@ -98,25 +125,24 @@ def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         with open(p) as f:
-            j = json.load(f)
-        return j, "measured"
+            return json.load(f), "measured"
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def gemm_traffic(workload, variant, schedule):
-    """DRAM bytes per tcgen05 GEMM launch from the committed ncu launch-list
-    summary of this workload (profiles/launches_<workload>_<variant>.md), or
-    None when there is none or when the GEMM sources changed since it was
-    captured (their SHA-256 is recorded next to the figure)."""
+def gemm_traffic(s, variant, schedule):
+    """Average DRAM bytes per tcgen05 GEMM launch of one full training step of
+    this workload, from the committed small-case ncu capture
+    (profiles/gemm_traffic_<workload>_<variant>.md: every GEMM launch of one
+    step of the same stack at depth 2, scaled to the full depth there), or None
+    when there is none, when the workload is not the one captured, or when the
+    GEMM sources changed since (their SHA-256 is recorded next to the figure)."""
     import hashlib
     import re
-    if schedule != "two_stream":
-        return None
-    path = os.path.join(ROOT, "profiles", f"launches_{workload}_{variant}.md")
-    if not os.path.exists(path):
+    path = os.path.join(ROOT, "profiles", f"gemm_traffic_{s.name}_{variant}.md")
+    if schedule != "two_stream" or not os.path.exists(path):
         return None
     text = open(path).read()
-    mb = re.search(r"^gemm_dram_bytes_per_launch:\s*(\d+)", text, re.M)
+    mb = re.search(r"^gemm_dram_bytes_per_launch_full_step:\s*(\d+)", text, re.M)
     mh = re.search(r"^gemm_sources_sha256:\s*([0-9a-f]{64})", text, re.M)
     if not mb or not mh:
         return None
@@ -127,31 +153,6 @@ def gemm_traffic(workload, variant, schedule):
     return int(mb.group(1)) if h.hexdigest() == mh.group(1) else None
 
 
-# ------------------------------------------------------------------ oracle arm
-def oracle_step_sample(s, variant, seed=1234):
-    """One fp64 oracle training step (forward, backward, AdamW) on a bounded
-    sample of the workload: full width and sequence, one layer, batch 1.
-    Returns (seconds, scale) where scale converts the sample's time into the
-    time of one full step by the ratio of algorithmic FLOPs."""
-    import numpy as np
-    from oracle import fal_oracle as O
-    sample = s.replace(layers=1, batch=1)
-    params = synth.init_params(variant, sample, seed)
-    tok, tgt = synth.make_tokens(sample, seed)
-    cfg = O.Config.from_shape(variant, sample)
-    hp = synth.adamw_hparams()
-    decayed = {n for n, _, dec in synth.param_specs(variant, sample) if dec}
-    zeros = {k: np.zeros(v.shape) for k, v in params.items()}
-    t0 = time.perf_counter()
-    _, cache = O.forward(params, cfg, tok, tgt)
-    grads = O.backward(params, cfg, cache)
-    O.adamw_step(params, grads, zeros, zeros, 1, hp["lr"], hp["beta1"], hp["beta2"], hp["eps"], hp["weight_decay"],
-                 decayed)
-    dt = time.perf_counter() - t0
-    scale = synth.model_flops_per_step(s) / synth.model_flops_per_step(sample)
-    return dt, scale
-
-
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -159,24 +160,76 @@ def cpu_cores():
         return os.cpu_count() or 1
 
 
+# ------------------------------------------------------------------ oracle
+class OracleSample:
+    """A measured, bounded sample of one training step of the stack `s`, run by
+    the fp64 oracle as it stands: forward and backward of `batch` sequences of
+    `seq` tokens at the full depth and width, plus AdamW on the same fraction
+    f = (batch * seq) / (s.batch * s.seq) of every parameter tensor (a
+    different slice of rows each call).  Every part of the step is thus timed
+    on f of its work, so tokens / time is the oracle's throughput on the
+    workload, apart from the causal attention, whose per-token cost grows with
+    the sequence (under 2 % of the FLOPs at the benchmark sequences).  The
+    seeded inputs are drawn once, and the parameters are held in fp64 so the
+    oracle's own conversion is the identity."""
+
+    def __init__(self, s, variant, batch, seq, seed=1234):
+        import numpy as np
+        from oracle import fal_oracle as O
+        self.O, self.np = O, np
+        self.sample = s.replace(batch=batch, seq=seq)
+        self.frac = self.sample.tokens / s.tokens
+        self.params = {k: v.astype(np.float64) for k, v in synth.init_params(variant, self.sample, seed).items()}
+        self.tok, self.tgt = synth.make_tokens(self.sample, seed)
+        self.cfg = O.Config.from_shape(variant, self.sample)
+        self.hp = synth.adamw_hparams()
+        self.decayed = {n for n, _, dec in synth.param_specs(variant, self.sample) if dec}
+        self.calls = 0
+
+    def __call__(self):
+        """Runs the sample; returns its wall time in seconds."""
+        O, hp, np = self.O, self.hp, self.np
+        nslices = max(1, round(1.0 / self.frac))
+        j = self.calls % nslices
+        self.calls += 1
+        t0 = time.perf_counter()
+        _, cache = O.forward(self.params, self.cfg, self.tok, self.tgt)
+        grads = O.backward(self.params, self.cfg, cache)
+        del cache
+        part = {}
+        for k, v in self.params.items():
+            r = v.shape[0]
+            lo, hi = j * r // nslices, (j + 1) * r // nslices
+            part[k] = slice(lo, hi)
+        sub = lambda d: {k: d[k][part[k]] for k in d}
+        zeros = {k: np.zeros_like(v) for k, v in sub(self.params).items()}
+        O.adamw_step(sub(self.params), sub(grads), zeros, zeros, 1, hp["lr"], hp["beta1"], hp["beta2"], hp["eps"],
+                     hp["weight_decay"], self.decayed)
+        return time.perf_counter() - t0
+
+    def describe(self, sec):
+        return (f"fp64 oracle on the host cores, measured: forward and backward of the full {self.sample.layers}-layer "
+                f"stack at full width on {self.sample.batch} sequence(s) of {self.sample.seq} tokens plus AdamW on the "
+                f"same fraction ({self.frac:.4g}) of every parameter tensor: {sec:.2f} s per sample")
+
+
 def run_reference(args, n):
+    """The reference arm: the fp64 oracle on the host cores.  Each step is a
+    measured OracleSample of the workload's step on one sequence of REF_SEQ
+    tokens; throughput = those tokens over the measured time."""
     s = shape_of(args)
+    step = OracleSample(s, args.variant, 1, min(REF_SEQ, s.seq))
     for _ in range(args.warmup):
-        oracle_step_sample(s, args.variant)
-    times = []
-    scale = 1.0
-    for _ in range(args.steps):
-        dt, scale = oracle_step_sample(s, args.variant)
-        times.append(dt * scale)
-    ms = statistics.mean(times) * 1e3
-    value = s.tokens / (ms / 1e3)
-    sample = (f"one step of the fp64 oracle per timed step on 1 of {s.layers} layers, batch 1 of {s.batch}, full width "
-              f"and seq; time scaled to the full step by the algorithmic FLOP ratio {scale:.1f}")
+        step()
+    times = [step() for _ in range(args.steps)]
+    sec = statistics.mean(times)
+    value = step.sample.tokens / sec
+    desc = "each timed step: " + step.describe(sec)
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": n, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+           "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": workload_config(s, args.variant, args.schedule, n),
-           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": desc},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
 
@@ -192,6 +245,7 @@ class ClockSampler:
     def __init__(self, index):
         self.proc = None
         self.index = index
+        self.out = ""
 
     def __enter__(self):
         try:
@@ -212,8 +266,6 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
                 self.out = ""
-        else:
-            self.out = ""
 
     def summary(self):
         rows = []
@@ -233,7 +285,7 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def init_flat_params(model, s, variant, seed, torch):
+def init_flat_params(model, s, seed, torch):
     """Seeded weights drawn on the device with the recipe of the synthetic-input
     module (N(0, 0.02), out-projections scaled when the shape asks for it,
     LN gamma = 1, beta = 0, zero biases)."""
@@ -254,59 +306,141 @@ def init_flat_params(model, s, variant, seed, torch):
     model.set_params(flat)
 
 
-def time_variant(args, s, variant, schedule, torch, fal, dev, n, world, rank, peaks, with_e2e):
-    hp = synth.adamw_hparams()
-    cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab, precision="bf16",
-                          schedule=schedule, **hp)
-    m = fal.Model(cfg, device=dev)
-    init_flat_params(m, s, variant, 1234 + rank, torch)
-    tok_np, tgt_np = synth.make_tokens(s, 1234 + rank)
-    tok = torch.from_numpy(tok_np).to(dev)
-    tgt = torch.from_numpy(tgt_np).to(dev)
-    for _ in range(args.warmup):
-        m.train_step(tok, tgt, sync=False)
-    loss0 = m.loss()
-    stream = m.stream_main
-    if world > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize(dev)
-    m.profile_enable(True)
-    n0 = fal.launch_count()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(torch.cuda.current_device()) as clk:
-        ev0.record(stream)
-        for _ in range(args.steps):
-            m.train_step(tok, tgt, sync=False)
-        ev1.record(stream)
-        torch.cuda.synchronize(dev)
-    launches = fal.launch_count() - n0
-    m.profile_enable(False)
-    prof = m.profile_read()
-    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, world, torch)
-    if world > 1:
-        torch.distributed.barrier()
-    loss1 = m.loss()
-    res = {"ms": ms, "launches": launches / args.steps * args.steps, "prof": prof, "clocks": clk.summary(),
-           "loss_first": loss0, "loss_last": loss1}
-    if with_e2e:
-        # Through the public C ABI with host buffers: pinned token upload, the
-        # step, and the loss read back every step.
-        tok_h = torch.from_numpy(tok_np).pin_memory()
-        tgt_h = torch.from_numpy(tgt_np).pin_memory()
-        m.train_step(tok_h, tgt_h, sync=True)
+class Arm:
+    """One model of the library on the device with its resident inputs."""
+
+    def __init__(self, s, variant, schedule, torch, fal, dev, rank):
+        hp = synth.adamw_hparams()
+        cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
+                              precision="bf16", schedule=schedule, **hp)
+        self.s, self.variant, self.schedule, self.torch, self.fal, self.dev = s, variant, schedule, torch, fal, dev
+        self.m = fal.Model(cfg, device=dev)
+        init_flat_params(self.m, s, 1234 + rank, torch)
+        self.tok_np, self.tgt_np = synth.make_tokens(s, 1234 + rank)
+        self.tok = torch.from_numpy(self.tok_np).to(dev)
+        self.tgt = torch.from_numpy(self.tgt_np).to(dev)
+
+    def steps(self, k):
+        for _ in range(k):
+            self.m.train_step(self.tok, self.tgt, sync=False)
+
+    def timed(self, steps, warmup, world, clocks=False):
+        """W untimed steps, then K steps between CUDA events on the library's
+        main stream (barrier + synchronize on both sides); max over ranks."""
+        torch = self.torch
+        self.steps(warmup)
         if world > 1:
             torch.distributed.barrier()
+        torch.cuda.synchronize(self.dev)
+        n0 = self.fal.launch_count()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        stream = self.m.stream_main
+        clk = ClockSampler(torch.cuda.current_device()) if clocks else None
+        if clk:
+            clk.__enter__()
+        ev0.record(stream)
+        self.steps(steps)
+        ev1.record(stream)
+        torch.cuda.synchronize(self.dev)
+        if clk:
+            clk.__exit__(None, None, None)
+        launches = self.fal.launch_count() - n0
+        ms = max_over_ranks(ev0.elapsed_time(ev1) / steps, world, torch)
+        if world > 1:
+            torch.distributed.barrier()
+        out = {"ms": ms, "launches": launches, "loss": self.m.loss()}
+        if clk:
+            out["clocks"] = clk.summary()
+        return out
+
+    def e2e(self, steps, world):
+        """Through the public C ABI with host buffers: pinned token upload, the
+        step, and the loss read back to the host every step."""
+        torch = self.torch
+        tok_h = torch.from_numpy(self.tok_np).pin_memory()
+        tgt_h = torch.from_numpy(self.tgt_np).pin_memory()
+        self.m.train_step(tok_h, tgt_h, sync=True)
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(self.dev)
         t0 = time.perf_counter()
-        for _ in range(args.steps):
-            m.train_step(tok_h, tgt_h, sync=True)
-        e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, world, torch)
-        res["e2e_s"] = e2e_s
-        res["h2d"] = tok_h.numel() * 4 * 2
-        res["d2h"] = 4
-    m.close()
-    del m
-    torch.cuda.empty_cache()
-    return res
+        for _ in range(steps):
+            self.m.train_step(tok_h, tgt_h, sync=True)
+        sec = max_over_ranks((time.perf_counter() - t0) / steps, world, torch)
+        return {"s": sec, "h2d": tok_h.numel() * 4 * 2, "d2h": 4}
+
+    def profiled(self, steps):
+        """GEMM and attention launches bracketed by CUDA events on their own
+        streams, over `steps` steps (a pass of its own, not the headline's)."""
+        self.torch.cuda.synchronize(self.dev)
+        self.m.profile_read()
+        self.m.profile_enable(True)
+        self.steps(steps)
+        prof = self.m.profile_read()
+        self.m.profile_enable(False)
+        return prof
+
+    def shares(self):
+        """Every launch of one step on its own CUDA events: time per kind."""
+        self.torch.cuda.synchronize(self.dev)
+        self.m.profile_read()
+        self.m.profile_enable(True, every_launch=True)
+        self.steps(1)
+        recs = self.m.profile_timeline()
+        self.m.profile_read()
+        self.m.profile_enable(False)
+        per = {}
+        for r in recs:
+            key = r["label"] or str(r["kind"])
+            e = per.setdefault(key, {"launches": 0, "ms": 0.0})
+            e["launches"] += 1
+            e["ms"] += r["end_ms"] - r["start_ms"]
+        span = (max(r["end_ms"] for r in recs) - min(r["start_ms"] for r in recs)) if recs else 0.0
+        return {"step_span_ms": span, "per_label": {k: {"launches": v["launches"], "ms": round(v["ms"], 4)}
+                                                    for k, v in sorted(per.items(), key=lambda kv: -kv[1]["ms"])}}
+
+    def close(self):
+        self.m.close()
+        del self.m
+        self.torch.cuda.empty_cache()
+
+
+def arm_summary(s, res, n, peaks):
+    flops = synth.model_flops_per_step(s)
+    tf = flops / (res["ms"] / 1e3) / 1e12
+    return {"value": job_throughput(s.tokens, n, res["ms"] / 1e3), "ms_per_step": res["ms"], "model_tflops": tf,
+            "frac_of_burst": tf / peaks.get("bf16_tflops", 1900.0),
+            "frac_of_sustained": tf / peaks.get("bf16_tflops_sustained", 1700.0)}
+
+
+def attention_isolated(s, torch, fal, dev):
+    """The attention kernels alone on one layer of the headline shape (CUDA
+    events, 3 warm-up and 10 timed launches each)."""
+    B, T, H, hd = s.batch, s.seq, s.heads, s.head_dim
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    qkv = torch.randn((B * T, 3 * H * hd), generator=g, device=dev).to(torch.bfloat16)
+    dctx = torch.randn((B * T, H * hd), generator=g, device=dev).to(torch.bfloat16)
+    ctx, lse = fal.attention_fwd(qkv, B, T, H, hd)
+
+    def clock(fn):
+        for _ in range(3):
+            fn()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        a.record()
+        for _ in range(10):
+            fn()
+        b.record()
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / 10
+
+    fwd_ms = clock(lambda: fal.attention_fwd(qkv, B, T, H, hd))
+    bwd_ms = clock(lambda: fal.attention_bwd(qkv, ctx, lse, dctx, B, T, H, hd))
+    f_fwd = 2.0 * B * H * T * T * hd  # causal half of 4*B*H*T^2*hd
+    return {"shape": f"B={B} T={T} H={H} hd={hd}", "fwd_us": fwd_ms * 1e3, "bwd_us": bwd_ms * 1e3,
+            "fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "bwd_tflops": 2 * f_fwd / (bwd_ms / 1e3) / 1e12,
+            "note": "backward includes its D = rowsum(dO*O) pre-pass; FLOPs algorithmic (backward = 2x forward)"}
 
 
 def main():
@@ -314,12 +448,15 @@ def main():
     world, rank, local = dist_env()
     n = max(world, 1)
     if world > 1:
-        import torch.distributed as td
         import torch
+        import torch.distributed as td
         td.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     if args.impl == "reference":
         if rank == 0:
             run_reference(args, n)
+        if world > 1:
+            import torch.distributed as td
+            td.destroy_process_group()
         return
 
     import torch
@@ -330,22 +467,23 @@ def main():
     dev = torch.device(f"cuda:{local}")
     fal.lib()
     peaks, peak_kind = measured_peaks()
-    s = shape_of(args)
-    main_res = time_variant(args, s, args.variant, args.schedule, torch, fal, dev, n, world, rank, peaks, True)
-    base = None
-    if not args.no_baseline and args.variant != "gpt":
-        base = time_variant(args, s, "gpt", "serial", torch, fal, dev, n, world, rank, peaks, False)
-
-    tokens = s.tokens * n
-    ms = main_res["ms"]
-    value = job_throughput(s.tokens, n, ms / 1e3)
-    flops = synth.model_flops_per_step(s)
     peak_burst = peaks.get("bf16_tflops", 1900.0)
     peak_sus = peaks.get("bf16_tflops_sustained", 1700.0)
+    s = shape_of(args)
+    flops = synth.model_flops_per_step(s)
+
+    # ---- headline (profiling off), end to end, then a separate profiled pass
+    arm = Arm(s, args.variant, args.schedule, torch, fal, dev, rank)
+    head = arm.timed(args.steps, args.warmup, world, clocks=True)
+    e2e = arm.e2e(args.steps, world)
+    prof = arm.profiled(min(args.steps, 3))
+    shares = arm.shares() if world == 1 else None
+    arm.close()
+    ms = head["ms"]
+    value = job_throughput(s.tokens, n, ms / 1e3)
     mfu = flops / (ms / 1e3) / 1e12
-    prof = main_res["prof"]
     gemm_tflops = prof["gemm_flops"] / (prof["gemm_ms"] / 1e3) / 1e12 if prof["gemm_ms"] > 0 else None
-    attn_tflops = prof["attn_flops"] / (prof["attn_ms"] / 1e3) / 1e12 if prof["attn_ms"] > 0 else None
+    psteps = min(args.steps, 3)
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": n, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
@@ -354,37 +492,72 @@ def main():
         "model_tflops": mfu,
         "frac_of_peak": {"burst": mfu / peak_burst, "sustained": mfu / peak_sus, "peak_kind": peak_kind},
         "roofline": {
-            "kernel": "gemm_tc2_kernel (tcgen05 GEMM on CTA pairs, all launches of the timed steps)",
+            "kernel": "gemm_tc2_kernel (tcgen05 GEMM on CTA pairs, every launch of the profiled steps)",
             "bound": "tensor", "achieved": gemm_tflops, "peak": peak_sus, "unit": "TFLOP/s",
             "frac": (gemm_tflops / peak_sus) if gemm_tflops else None,
-            "traffic": gemm_traffic(args.workload if args.layers is None and args.batch is None else "",
-                                    args.variant, args.schedule),
-            "traffic_unit": "DRAM bytes per launch (ncu launch list of this workload, profiles/)",
-            "peak_kind": f"{peak_kind} bf16_tflops_sustained (kernel timed inside a long step)",
-            "launches_per_step": prof["gemm_launches"] / args.steps,
-            "time_share_of_step": prof["gemm_ms"] / (ms * args.steps),
+            "frac_of_burst": (gemm_tflops / peak_burst) if gemm_tflops else None,
+            "traffic": gemm_traffic(s, args.variant, args.schedule),
+            "traffic_unit": "DRAM bytes per launch, average over one full step (small-case ncu capture, profiles/)",
+            "peak_kind": f"{peak_kind} bf16_tflops_sustained (kernel timed inside a long step); "
+                         f"frac_of_burst against bf16_tflops",
+            "launches_per_step": prof["gemm_launches"] / psteps,
+            "gemm_ms_per_step": prof["gemm_ms"] / psteps,
+            "profiled_steps": psteps,
         },
-        "attention": {"achieved_tflops": attn_tflops, "ms_per_step": prof["attn_ms"] / args.steps,
-                      "launches_per_step": prof["attn_launches"] / args.steps},
-        "gpu_launches": int(main_res["launches"]),
-        "clocks": main_res["clocks"],
-        "loss": {"after_warmup": main_res["loss_first"], "after_timed": main_res["loss_last"]},
+        "attention_in_step": {"ms_per_step": prof["attn_ms"] / psteps, "launches_per_step": prof["attn_launches"] / psteps,
+                              "note": "event time on the side stream while other kernels share the SMs"},
+        "gpu_launches": int(head["launches"]),
+        "clocks": head["clocks"],
+        "loss": {"after_timed": head["loss"]},
+        "e2e": {"value": job_throughput(s.tokens, n, e2e["s"]), "unit": UNIT, "h2d_bytes_per_step": e2e["h2d"],
+                "d2h_bytes_per_step": e2e["d2h"]},
     }
-    e2e_s = main_res.get("e2e_s")
-    out["e2e"] = {"value": tokens / e2e_s, "unit": UNIT, "h2d_bytes_per_step": main_res["h2d"],
-                  "d2h_bytes_per_step": main_res["d2h"]}
-    if base is not None:
-        gv = tokens / (base["ms"] / 1e3)
-        out["gpt_baseline"] = {"value": gv, "ms_per_step": base["ms"], "model_tflops": flops / (base["ms"] / 1e3) / 1e12,
-                               "schedule": "serial"}
-        out["speedup_vs_gpt"] = value / gv
+    if shares:
+        out["step_shares"] = shares
+    extra = world == 1
+    if extra:
+        out["attention_isolated"] = attention_isolated(s, torch, fal, dev)
+    k, w = args.arm_steps, min(args.warmup, 3)
+    if not args.no_baseline and extra:
+        if args.variant != "gpt":
+            a = Arm(s, args.variant, "serial", torch, fal, dev, rank)
+            r = a.timed(k, w, world)
+            a.close()
+            out["fal_serial" if args.variant == "fal" else f"{args.variant}_serial"] = dict(
+                arm_summary(s, r, n, peaks), schedule="serial")
+            if args.variant == "fal" and args.schedule == "two_stream":
+                out["two_stream_gain"] = r["ms"] / ms
+        a = Arm(s, "gpt", "serial", torch, fal, dev, rank)
+        r = a.timed(k, w, world)
+        a.close()
+        out["gpt_baseline"] = dict(arm_summary(s, r, n, peaks), schedule="serial")
+        out["speedup_vs_gpt"] = out["gpt_baseline"]["ms_per_step"] / ms
+    if not args.no_configs and extra and args.layers is None and args.batch is None:
+        cfgs = {}
+        for name, variants in CONFIG_ARMS:
+            if name == s.name:
+                continue
+            cs = synth.SHAPES[name]
+            row = {}
+            for v in variants:
+                sched = "two_stream" if v == "fal" else "serial"
+                a = Arm(cs, v, sched, torch, fal, dev, rank)
+                r = a.timed(k, w, world)
+                a.close()
+                row[variant_name(v)] = dict(arm_summary(cs, r, n, peaks), schedule=sched)
+            for v in variants:
+                if v != "gpt":
+                    row[f"{variant_name(v)}/GPT"] = row["GPT"]["ms_per_step"] / row[variant_name(v)]["ms_per_step"]
+            row["shape"] = (f"L={cs.layers} d_model={cs.d_model} heads={cs.heads} d_ff={cs.d_ff} seq={cs.seq} "
+                            f"batch={cs.batch} vocab={cs.vocab}")
+            cfgs[name] = row
+        out["configs"] = cfgs
+        out["configs_note"] = f"{w} warm-up and {k} timed steps per arm; fractions against measured burst / sustained"
     if rank == 0 and n == 1 and not args.no_cpu:
-        dt, scale = oracle_step_sample(s, args.variant)
-        cpu_val = s.tokens / (dt * scale)
-        out["cpu_baseline"] = {
-            "value": cpu_val, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-            "sample": f"one fp64 oracle step (forward, backward, AdamW) on 1 of {s.layers} layers, batch 1, full width "
-                      f"and seq ({dt:.1f} s), scaled to the full step by the algorithmic FLOP ratio {scale:.1f}"}
+        cpu = OracleSample(s, args.variant, 1, min(CPU_SEQ, s.seq))
+        sec = cpu()
+        out["cpu_baseline"] = {"value": cpu.sample.tokens / sec, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                               "sample": cpu.describe(sec)}
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:

@@ -128,6 +128,15 @@ int fal_set_params(fal_handle* h, const float* src, size_t n);
 int fal_get_params(fal_handle* h, float* dst, size_t n);
 int fal_get_grads(fal_handle* h, float* dst, size_t n);
 
+/* AdamW state, for checkpoint / resume: the first and second moments (flat
+ * fp32 buffers laid out like the parameters, n == n_elems; src/dst device or
+ * host, either pointer may be NULL to skip that buffer) and the number of
+ * optimizer steps taken so far (the next step's bias corrections use
+ * step + 1).  fal_set_opt_state does not touch the parameters; call it after
+ * fal_set_params, which resets the state to zero. */
+int fal_get_opt_state(fal_handle* h, float* m, float* v, size_t n, long long* step);
+int fal_set_opt_state(fal_handle* h, const float* m, const float* v, size_t n, long long step);
+
 /* Debug view of a saved activation of the last forward, converted to fp32.
  * name in {"X","u","m","qkv","ctx","h","g","Y","a1","xf","logits"}; layer is
  * ignored for the global ones ("a1","xf","logits"; "X" with layer==L is the

@@ -25,7 +25,9 @@
 //               from there as their A operand (so only B comes from shared
 //               memory, whose bandwidth bounds these small-N products).  At
 //               the end they scale and store dK, dV or dQ in bf16.
-// D = rowsum(dO * O) comes from a separate small kernel.  Every mbarrier wait
+// D = rowsum(dO * O) is an input: in the model it comes from the epilogue of the
+// GEMM that produces dO, at the kernel-level entry points from a small pre-pass
+// kernel (attention.cu).  Every mbarrier wait
 // is bounded; on expiry the kernel records DEV_ERR_TIMEOUT, lets its MMAs
 // finish, frees TMEM and returns.
 #include <cstring>

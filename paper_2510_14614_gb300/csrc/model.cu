@@ -1030,6 +1030,31 @@ int fal_get_grads(fal_handle* h, float* dst, size_t n) {
   return FAL_OK;
 }
 
+int fal_get_opt_state(fal_handle* h, float* m, float* v, size_t n, long long* step) {
+  if (!h) return FAL_ERR_ARG;
+  if (n != h->n_params) return fail(h, FAL_ERR_ARG, "parameter count mismatch");
+  int r = read_dev_err(h);
+  if (r) return r;
+  if ((m && cudaMemcpy(m, h->Mo, n * 4, cudaMemcpyDefault) != cudaSuccess) ||
+      (v && cudaMemcpy(v, h->Vo, n * 4, cudaMemcpyDefault) != cudaSuccess))
+    return fail(h, FAL_ERR_CUDA, "copy failed");
+  if (step) *step = h->step_t;
+  return FAL_OK;
+}
+
+int fal_set_opt_state(fal_handle* h, const float* m, const float* v, size_t n, long long step) {
+  if (!h) return FAL_ERR_ARG;
+  if (n != h->n_params) return fail(h, FAL_ERR_ARG, "parameter count mismatch");
+  if (step < 0) return fail(h, FAL_ERR_ARG, "negative step count");
+  cudaStream_t s = h->sm;
+  if ((m && cudaMemcpyAsync(h->Mo, m, n * 4, cudaMemcpyDefault, s) != cudaSuccess) ||
+      (v && cudaMemcpyAsync(h->Vo, v, n * 4, cudaMemcpyDefault, s) != cudaSuccess) ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return fail(h, FAL_ERR_CUDA, "copy failed");
+  h->step_t = (long)step;
+  return FAL_OK;
+}
+
 int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n) {
   if (!h || !name || !dst) return FAL_ERR_ARG;
   const std::string nm = name;

@@ -67,6 +67,10 @@ _SIGS = {
     "fal_set_params": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t]),
     "fal_get_params": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t]),
     "fal_get_grads": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t]),
+    "fal_get_opt_state": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                         ctypes.POINTER(ctypes.c_longlong)]),
+    "fal_set_opt_state": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
+                                         ctypes.c_longlong]),
     "fal_get_tap": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t]),
     "fal_profile_enable": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int]),
     "fal_profile_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(FalProfile)]),
@@ -198,6 +202,20 @@ class Model:
 
     def grads(self):
         return self.unflatten(self._flat(lib().fal_get_grads))
+
+    def opt_state(self):
+        """(m, v, step): AdamW moments as dicts name -> array, and the steps taken."""
+        m = np.empty(self.n_params, np.float32)
+        v = np.empty(self.n_params, np.float32)
+        step = ctypes.c_longlong()
+        _check(lib().fal_get_opt_state(self.h, m.ctypes.data_as(ctypes.c_void_p), v.ctypes.data_as(ctypes.c_void_p),
+                                       self.n_params, ctypes.byref(step)), self.h, "fal_get_opt_state")
+        return self.unflatten(m), self.unflatten(v), step.value
+
+    def set_opt_state(self, m: dict, v: dict, step: int):
+        fm, fv = self.flatten(m), self.flatten(v)
+        _check(lib().fal_set_opt_state(self.h, fm.ctypes.data_as(ctypes.c_void_p), fv.ctypes.data_as(ctypes.c_void_p),
+                                       self.n_params, int(step)), self.h, "fal_set_opt_state")
 
     # ------------------------------------------------------------- training
     def _tokens(self, tokens, targets):
