@@ -23,7 +23,22 @@ NumPy (matmul is the only library primitive used):
     attention scale 1/sqrt(head_dim), causal mask (key j visible to query t
     iff j <= t), mean token cross-entropy.
   * AdamW (App. A: lr 1e-4, weight decay 1e-3) with bias correction and
-    decoupled weight decay on matrices and embeddings.
+    decoupled weight decay on matrices and embeddings; gradient clipping to a
+    global L2 norm (App. A clips at 1).
+  * The paper's comparison blocks:
+      - Parallel (Sec. 5.1 baselines; GPT-J style): X_i + MHA_i(LN(X_i)) +
+        MLP_i(LN(X_i)), one LayerNorm feeding both branches;
+      - Ablation1 (App. D): X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i) +
+        LN(MHA_i(LN(X_i)))), the FAL structure with the block's own attention
+        and a LayerNorm LN_{A,i} of its own on it, every block;
+      - Ablation2 (App. D): block 1 is the standard block (its printed
+        equation drops a parenthesis, read like FAL+'s block 1), every later
+        block is the Parallel block;
+      - FAL+ reusing block k (App. D "Ablation with Other Layers"): blocks 1..k
+        are standard, block i > k adds LN_{F,i}(MHA_k(LN(X_k))); k = 1 is FAL+;
+      - FAL with a separate LayerNorm on X_i for the MLP input
+        (``separate_ln2``): the other reading of Eq. 2's MLP input, kept here
+        only to show that the reading matters.
 
 Parameters are a dict name -> array (names from the shared synthetic-input
 module); weight matrices are [out, in].  Parity pins for every function here
@@ -106,16 +121,22 @@ def cross_entropy(logits, targets):
 
 
 # ---------------------------------------------------------------- the model
+VARIANTS = ("gpt", "fal", "falplus", "parallel", "ablation1", "ablation2")
+
+
 class Config:
-    def __init__(self, variant, layers, d_model, heads, d_ff, seq, batch, vocab):
-        assert variant in ("gpt", "fal", "falplus")
+    def __init__(self, variant, layers, d_model, heads, d_ff, seq, batch, vocab, reuse=1, separate_ln2=False):
+        assert variant in VARIANTS
         assert d_model % heads == 0
+        assert reuse >= 1 and (reuse == 1 or variant == "falplus")
+        assert not separate_ln2 or variant == "fal"
         self.variant, self.layers, self.d_model, self.heads = variant, layers, d_model, heads
         self.d_ff, self.seq, self.batch, self.vocab = d_ff, seq, batch, vocab
+        self.reuse, self.separate_ln2 = reuse, separate_ln2
 
     @classmethod
-    def from_shape(cls, variant, s):
-        return cls(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab)
+    def from_shape(cls, variant, s, **kw):
+        return cls(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab, **kw)
 
 
 def _split_heads(x, B, T, H):
@@ -138,7 +159,8 @@ def forward(params, cfg, tokens, targets, layers=None):
     var = cfg.variant
     X = (P["wte"][tokens] + P["wpe"][:T][None]).reshape(B * T, d)
     cache = {"X": [X], "layers": []}
-    a1 = None
+    a1 = None    # first attention output (FAL), or block k's (FAL+ reusing k)
+    k_reuse = cfg.reuse - 1
     for i in range(L):
         w = lambda n: P[f"h{i}.{n}"]
         c = {}
@@ -148,17 +170,26 @@ def forward(params, cfg, tokens, targets, layers=None):
         o, p = causal_attention(q, k, v)
         ctx = _merge_heads(o)
         a = ctx @ w("attn.w_o").T + w("attn.b_o")
-        if i == 0:
+        if i == k_reuse:
             a1 = a
         if var == "fal":
             if i == 0:
                 cache["F"], cache["lnF"] = layer_norm(a1, P["lnF.g"], P["lnF.b"])
-            m = u + cache["F"]
-        else:
+            if cfg.separate_ln2:
+                m, c["ln2"] = layer_norm(X, w("ln2.g"), w("ln2.b"))
+                m = m + cache["F"]
+            else:
+                m = u + cache["F"]
+        elif var == "parallel" or (var == "ablation2" and i >= 1):
+            m = u
+        elif var == "ablation1":
+            fa, c["lnA"] = layer_norm(a, w("lnA.g"), w("lnA.b"))
+            m = u + fa
+        else:  # gpt, falplus, block 1 of ablation2
             Y = X + a
             m, c["ln2"] = layer_norm(Y, w("ln2.g"), w("ln2.b"))
             c["Y"] = Y
-            if var == "falplus" and i >= 1:
+            if var == "falplus" and i > k_reuse:
                 fa, c["lnF"] = layer_norm(a1, w("lnF.g"), w("lnF.b"))
                 m = m + fa
         h = m @ w("mlp.w_up").T + w("mlp.b_up")
@@ -188,7 +219,8 @@ def backward(params, cfg, cache):
     dX, G["lnf.g"], G["lnf.b"] = layer_norm_backward(dxf, cache["lnf"], P["lnf.g"])
 
     dF = np.zeros((B * T, d))   # FAL: gradient reaching F = LN_F(a_1)
-    da1 = np.zeros((B * T, d))  # FAL+: gradient reaching a_1 through LN_{F,i}
+    da1 = np.zeros((B * T, d))  # FAL+: gradient reaching a_1 (or a_k) through LN_{F,i}
+    k_reuse = cfg.reuse - 1
     for i in reversed(range(L)):
         c = cache["layers"][i]
         w = lambda n: P[f"h{i}.{n}"]
@@ -204,21 +236,30 @@ def backward(params, cfg, cache):
         dm = dh @ w("mlp.w_up")
         du = np.zeros((B * T, d))
         if var == "fal":
-            du += dm
+            if cfg.separate_ln2:
+                dx2, G[gn("ln2.g")], G[gn("ln2.b")] = layer_norm_backward(dm, c["ln2"], w("ln2.g"))
+                dXi += dx2
+            else:
+                du += dm
             dF += dm
+        elif var == "parallel" or (var == "ablation2" and i >= 1):
+            du += dm
+        elif var == "ablation1":
+            du += dm
+            dfa, G[gn("lnA.g")], G[gn("lnA.b")] = layer_norm_backward(dm, c["lnA"], w("lnA.g"))
+            da += dfa
         else:
             dY, G[gn("ln2.g")], G[gn("ln2.b")] = layer_norm_backward(dm, c["ln2"], w("ln2.g"))
             dXi += dY
             da += dY
-            if var == "falplus" and i >= 1:
+            if var == "falplus" and i > k_reuse:
                 dfa, G[gn("lnF.g")], G[gn("lnF.b")] = layer_norm_backward(dm, c["lnF"], w("lnF.g"))
                 da1 += dfa
-        if i == 0:
-            if var == "fal":
-                dfa, G["lnF.g"], G["lnF.b"] = layer_norm_backward(dF, cache["lnF"], P["lnF.g"])
-                da += dfa
-            elif var == "falplus":
-                da += da1
+        if var == "fal" and i == 0:
+            dfa, G["lnF.g"], G["lnF.b"] = layer_norm_backward(dF, cache["lnF"], P["lnF.g"])
+            da += dfa
+        if var == "falplus" and i == k_reuse:
+            da += da1
         G[gn("attn.w_o")] = da.T @ c["ctx"]
         G[gn("attn.b_o")] = da.sum(0)
         dctx = _split_heads(da @ w("attn.w_o"), B, T, H)
@@ -233,6 +274,16 @@ def backward(params, cfg, cache):
     np.add.at(G["wte"], tok, dX)
     G["wpe"][:T] += dX.reshape(B, T, d).sum(0)
     return G
+
+
+def clip_grad_norm(grads, max_norm):
+    """Gradient clipping by the global L2 norm over every tensor (App. A clips
+    at 1.0): when the norm exceeds max_norm every gradient is scaled by
+    max_norm / norm.  Returns the clipped gradients and the norm before
+    clipping."""
+    norm = math.sqrt(sum(float(np.sum(np.asarray(g, np.float64) ** 2)) for g in grads.values()))
+    scale = max_norm / norm if norm > max_norm else 1.0
+    return {k: np.asarray(g, np.float64) * scale for k, g in grads.items()}, norm
 
 
 def adamw_step(params, grads, m, v, t, lr, beta1, beta2, eps, weight_decay, decayed):

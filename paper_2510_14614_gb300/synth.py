@@ -24,6 +24,9 @@ import math
 import numpy as np
 
 VARIANTS = ("gpt", "fal", "falplus")
+# The paper's comparison blocks (Sec. 5.1 baselines, App. D ablations).
+COMPARISON_VARIANTS = ("parallel", "ablation1", "ablation2")
+ALL_VARIANTS = VARIANTS + COMPARISON_VARIANTS
 
 
 @dataclasses.dataclass(frozen=True)
@@ -70,15 +73,20 @@ def model_flops_per_step(s: Shape) -> float:
     return 6.0 * bt * (L * (4 * d * d + 2 * d * f) + d * s.vocab) + 6.0 * bt * L * s.seq * d
 
 
-def param_specs(variant: str, s: Shape):
+def param_specs(variant: str, s: Shape, reuse: int = 1, separate_ln2: bool = False):
     """Canonical list of (name, shape, decayed) for a variant and shape.
 
     Layers are numbered from 0 (the paper's block 1 is ``h0``).  Weight
     matrices are stored [out, in].  Weight decay applies to matrices and
-    embeddings only.
+    embeddings only.  ``reuse`` (FAL+ only) is the paper's index k >= 1 of the
+    block whose attention output later blocks add; blocks after it carry their
+    own LayerNorm ``lnF`` on it.  ``separate_ln2`` (FAL only) gives every block
+    a LayerNorm ``ln2`` of its own for the MLP input.
     """
-    if variant not in VARIANTS:
+    if variant not in ALL_VARIANTS:
         raise ValueError(f"unknown variant {variant!r}")
+    if reuse < 1 or (reuse != 1 and variant != "falplus") or (separate_ln2 and variant != "fal"):
+        raise ValueError("reuse applies to FAL+ and separate_ln2 to FAL")
     d, f, V, T, L = s.d_model, s.d_ff, s.vocab, s.seq, s.layers
     specs = [("wte", (V, d), True), ("wpe", (T, d), True)]
     for i in range(L):
@@ -88,10 +96,12 @@ def param_specs(variant: str, s: Shape):
             (p + "attn.w_qkv", (3 * d, d), True), (p + "attn.b_qkv", (3 * d,), False),
             (p + "attn.w_o", (d, d), True), (p + "attn.b_o", (d,), False),
         ]
-        if variant in ("gpt", "falplus"):
+        if variant in ("gpt", "falplus") or (variant == "ablation2" and i == 0) or separate_ln2:
             specs += [(p + "ln2.g", (d,), False), (p + "ln2.b", (d,), False)]
-        if variant == "falplus" and i >= 1:
+        if variant == "falplus" and i >= reuse:
             specs += [(p + "lnF.g", (d,), False), (p + "lnF.b", (d,), False)]
+        if variant == "ablation1":
+            specs += [(p + "lnA.g", (d,), False), (p + "lnA.b", (d,), False)]
         specs += [
             (p + "mlp.w_up", (f, d), True), (p + "mlp.b_up", (f,), False),
             (p + "mlp.w_down", (d, f), True), (p + "mlp.b_down", (d,), False),
@@ -102,11 +112,11 @@ def param_specs(variant: str, s: Shape):
     return specs
 
 
-def init_params(variant: str, s: Shape, seed: int = 0, std: float = 0.02):
+def init_params(variant: str, s: Shape, seed: int = 0, std: float = 0.02, **spec_kw):
     """Seeded N(0, std) weights (fp64 draw rounded to fp32), LN gamma=1/beta=0, zero biases."""
     rng = np.random.default_rng([seed, 1])
     out = {}
-    for name, shape, _ in param_specs(variant, s):
+    for name, shape, _ in param_specs(variant, s, **spec_kw):
         leaf = name.rsplit(".", 1)[-1]
         if name in ("wte", "wpe") or leaf.startswith("w_"):
             sd = std

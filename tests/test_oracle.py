@@ -309,3 +309,166 @@ def test_fal_with_zero_first_attention_ln_is_parallel_block():
     assert abs(loss - tl) < 1e-12
     for k, g in tg.items():
         np.testing.assert_allclose(grads[k], g, rtol=1e-9, atol=1e-13, err_msg=k)
+
+
+# ------------------------------------------------------------------ comparison blocks
+# (variant, oracle/spec options) for the paper's comparison blocks and readings
+COMPARISONS = [("parallel", {}), ("ablation1", {}), ("ablation2", {}), ("falplus", {"reuse": 2}),
+               ("falplus", {"reuse": 3}), ("fal", {"separate_ln2": True})]
+CMP_IDS = [v + "".join(f"-{k}{int(x)}" for k, x in kw.items()) for v, kw in COMPARISONS]
+
+
+def _cparams(variant, kw, s, seed):
+    return synth.perturb_params(synth.init_params(variant, s, seed, **kw), seed)
+
+
+@pytest.mark.parametrize("variant,kw", COMPARISONS, ids=CMP_IDS)
+def test_comparison_blocks_match_autograd_model(variant, kw):
+    s = TINY.replace(layers=3)
+    p = _cparams(variant, kw, s, 21)
+    tok, tgt = synth.make_tokens(s, 5)
+    cfg = O.Config.from_shape(variant, s, **kw)
+    loss, cache = O.forward(p, cfg, tok, tgt)
+    grads = O.backward(p, cfg, cache)
+    tloss, tgrads = torch_ref.loss_and_grads(p, variant, s.heads, tok, tgt, s.layers, **kw)
+    assert abs(loss - tloss) < 1e-12
+    assert set(grads) == set(p)
+    for k in p:
+        np.testing.assert_allclose(grads[k], tgrads[k], rtol=1e-9, atol=1e-13, err_msg=k)
+
+
+@pytest.mark.parametrize("variant,kw", COMPARISONS, ids=CMP_IDS)
+def test_comparison_blocks_backward_matches_central_differences(variant, kw):
+    s = TINY.replace(layers=3)
+    p = {k: a.astype(np.float64) for k, a in _cparams(variant, kw, s, 22).items()}
+    tok, tgt = synth.make_tokens(s, 6)
+    cfg = O.Config.from_shape(variant, s, **kw)
+    _, cache = O.forward(p, cfg, tok, tgt)
+    grads = O.backward(p, cfg, cache)
+    rng = np.random.default_rng(23)
+    h = 1e-5
+    for k in p:
+        direction = rng.standard_normal(p[k].shape)
+        direction /= np.linalg.norm(direction)
+        pp, pm = dict(p), dict(p)
+        pp[k], pm[k] = p[k] + h * direction, p[k] - h * direction
+        fd = (O.loss_only(pp, cfg, tok, tgt) - O.loss_only(pm, cfg, tok, tgt)) / (2 * h)
+        an = float((grads[k] * direction).sum())
+        assert abs(fd - an) <= 1e-6 * np.linalg.norm(grads[k]) + 1e-11, (k, fd, an)
+
+
+def _run(variant, p, s, tok, tgt, **kw):
+    cfg = O.Config.from_shape(variant, s, **kw)
+    loss, cache = O.forward(p, cfg, tok, tgt)
+    return loss, cache, O.backward(p, cfg, cache)
+
+
+def test_ablation1_with_zero_own_attention_ln_is_parallel():
+    """Ablation1 (App. D) adds LN_{A,i}(MHA_i) to the MLP input; with every
+    LN_{A,i} switched off it is the Parallel block."""
+    s = TINY.replace(layers=3)
+    p = _cparams("ablation1", {}, s, 24)
+    for i in range(s.layers):
+        p[f"h{i}.lnA.g"] = np.zeros_like(p[f"h{i}.lnA.g"])
+        p[f"h{i}.lnA.b"] = np.zeros_like(p[f"h{i}.lnA.b"])
+    q = {k: v for k, v in p.items() if ".lnA." not in k}
+    tok, tgt = synth.make_tokens(s, 7)
+    la, _, ga = _run("ablation1", p, s, tok, tgt)
+    lp, _, gp = _run("parallel", q, s, tok, tgt)
+    assert la == lp
+    for k in q:
+        np.testing.assert_array_equal(ga[k], gp[k], err_msg=k)
+
+
+def test_ablation1_mlp_input_follows_own_attention():
+    """Unlike FAL, Ablation1's MLP input in block i reads MHA_i: changing block
+    2's attention weights changes block 2's MLP input."""
+    s = TINY.replace(layers=3)
+    p = _cparams("ablation1", {}, s, 25)
+    q = dict(p, **{"h1.attn.w_o": p["h1.attn.w_o"] * 1.5})
+    tok, tgt = synth.make_tokens(s, 8)
+    _, c0, _ = _run("ablation1", p, s, tok, tgt)
+    _, c1, _ = _run("ablation1", q, s, tok, tgt)
+    np.testing.assert_array_equal(c0["layers"][1]["u"], c1["layers"][1]["u"])
+    assert not np.allclose(c0["layers"][1]["m"], c1["layers"][1]["m"])
+
+
+def test_ablation2_first_block_is_gpt_later_blocks_are_parallel():
+    """Ablation2 (App. D) keeps only block 1's MHA-MLP connection: its block 1
+    is the GPT block and every later block the Parallel block."""
+    s = TINY.replace(layers=3)
+    p = _cparams("ablation2", {}, s, 26)
+    tok, tgt = synth.make_tokens(s, 9)
+    _, c, _ = _run("ablation2", p, s, tok, tgt)
+    g1 = {k: v for k, v in p.items() if not k.startswith(("h1.", "h2."))}
+    _, cg, _ = _run("gpt", g1, s.replace(layers=1), tok, tgt)
+    np.testing.assert_array_equal(c["X"][1], cg["X"][1])
+    for i in (1, 2):
+        np.testing.assert_array_equal(c["layers"][i]["m"], c["layers"][i]["u"])
+
+
+def test_falplus_reuse_first_block_is_falplus_and_earlier_blocks_are_gpt():
+    """FAL+ reusing block k: k = 1 is FAL+; blocks 1..k are standard blocks
+    (GPT through X_{k+1}); with every LN_{F,i} switched off it is GPT."""
+    s = TINY.replace(layers=3)
+    tok, tgt = synth.make_tokens(s, 10)
+    p1 = _cparams("falplus", {}, s, 27)
+    l_a, _, g_a = _run("falplus", p1, s, tok, tgt)
+    l_b, _, g_b = _run("falplus", p1, s, tok, tgt, reuse=1)
+    assert l_a == l_b
+    p2 = _cparams("falplus", {"reuse": 2}, s, 27)
+    _, c2, _ = _run("falplus", p2, s, tok, tgt, reuse=2)
+    pg = {k: v for k, v in p2.items() if ".lnF." not in k}
+    _, cg, gg = _run("gpt", pg, s, tok, tgt)
+    np.testing.assert_array_equal(c2["X"][2], cg["X"][2])
+    np.testing.assert_array_equal(c2["a1"], cg["layers"][1]["a"])
+    assert not np.allclose(c2["X"][3], cg["X"][3])
+    z = dict(p2, **{"h2.lnF.g": np.zeros_like(p2["h2.lnF.g"]), "h2.lnF.b": np.zeros_like(p2["h2.lnF.b"])})
+    lz, _, gz = _run("falplus", z, s, tok, tgt, reuse=2)
+    lg, _, _ = _run("gpt", pg, s, tok, tgt)
+    assert lz == lg
+    for k in pg:
+        np.testing.assert_allclose(gz[k], gg[k], rtol=1e-12, atol=1e-15, err_msg=k)
+
+
+def test_separate_ln2_reading_of_fal():
+    """The other reading of Eq. 2's MLP input (a LayerNorm of its own on X_i)
+    equals the adopted one when that LayerNorm has LN1's parameters, and
+    differs from it otherwise: the reading is observable."""
+    s = TINY.replace(layers=3)
+    tok, tgt = synth.make_tokens(s, 11)
+    p = _cparams("fal", {}, s, 28)
+    q = dict(p)
+    for i in range(s.layers):
+        q[f"h{i}.ln2.g"], q[f"h{i}.ln2.b"] = p[f"h{i}.ln1.g"], p[f"h{i}.ln1.b"]
+    l0, _, _ = _run("fal", p, s, tok, tgt)
+    l1, _, g1 = _run("fal", q, s, tok, tgt, separate_ln2=True)
+    assert abs(l0 - l1) < 1e-13
+    r = dict(q, **{"h1.ln2.b": q["h1.ln2.b"] + 0.3})
+    l2, _, _ = _run("fal", r, s, tok, tgt, separate_ln2=True)
+    assert abs(l2 - l0) > 1e-6
+    # with LN2 tied to LN1, LN1's gradient under the shared reading is the sum of both
+    _, _, g0 = _run("fal", p, s, tok, tgt)
+    for i in range(s.layers):
+        np.testing.assert_allclose(g1[f"h{i}.ln1.g"] + g1[f"h{i}.ln2.g"], g0[f"h{i}.ln1.g"], rtol=1e-9, atol=1e-13)
+
+
+@pytest.mark.parametrize("max_norm", [1.0, 1e-3, 1e6])
+def test_clip_grad_norm_matches_torch(max_norm):
+    rng = np.random.default_rng(29)
+    grads = {"a": rng.standard_normal((5, 7)), "b": rng.standard_normal(11) * 3}
+    clipped, norm = O.clip_grad_norm(grads, max_norm)
+    ts = [torch.zeros(g.shape, requires_grad=True) for g in grads.values()]
+    for t, g in zip(ts, grads.values()):
+        t.grad = torch.tensor(g)
+    tn = torch.nn.utils.clip_grad_norm_(ts, max_norm)
+    assert abs(norm - float(tn)) < 1e-12 * norm
+    for t, k in zip(ts, grads):
+        # torch divides by norm + 1e-6; the clipping definition divides by the norm
+        np.testing.assert_allclose(clipped[k], t.grad.numpy(), rtol=2e-6 / max(min(norm, max_norm), 1e-30) + 1e-14)
+    if norm <= max_norm:
+        for k in grads:
+            np.testing.assert_array_equal(clipped[k], grads[k])
+    else:
+        total = math.sqrt(sum(float((c ** 2).sum()) for c in clipped.values()))
+        assert abs(total - max_norm) < 1e-12 * max_norm

@@ -32,9 +32,12 @@ def _mlp(x, p, i):
     return Fn.linear(Fn.gelu(h, approximate="tanh"), p[f"h{i}.mlp.w_down"], p[f"h{i}.mlp.b_down"])
 
 
-def model_loss(params, variant, heads, tokens, targets, layers, parallel=False):
+def model_loss(params, variant, heads, tokens, targets, layers, parallel=False, reuse=1, separate_ln2=False):
     """Mean next-token loss.  ``parallel=True`` builds the GPT-J style block
-    X + MHA(LN1(X)) + MLP(LN1(X)) (no first-attention term)."""
+    X + MHA(LN1(X)) + MLP(LN1(X)) (no first-attention term), as does the
+    variant "parallel"; "ablation1" / "ablation2" are App. D's ablations;
+    ``reuse`` = k makes FAL+ add block k's attention; ``separate_ln2`` gives
+    FAL's MLP input a LayerNorm of its own."""
     p = params
     tok = torch.as_tensor(tokens, dtype=torch.long)
     B, T = tok.shape
@@ -43,15 +46,17 @@ def model_loss(params, variant, heads, tokens, targets, layers, parallel=False):
     for i in range(layers):
         n1 = _ln(X, p, f"h{i}.ln1")
         a = _mha(n1, p, i, heads)
-        if i == 0:
+        if i == reuse - 1:
             a1 = a
-        if parallel:
+        if parallel or variant == "parallel" or (variant == "ablation2" and i >= 1):
             m = n1
+        elif variant == "ablation1":
+            m = n1 + _ln(a, p, f"h{i}.lnA")
         elif variant == "fal":
-            m = n1 + _ln(a1, p, "lnF")
+            m = (_ln(X, p, f"h{i}.ln2") if separate_ln2 else n1) + _ln(a1, p, "lnF")
         else:
             m = _ln(X + a, p, f"h{i}.ln2")
-            if variant == "falplus" and i >= 1:
+            if variant == "falplus" and i >= reuse:
                 m = m + _ln(a1, p, f"h{i}.lnF")
         X = X + a + _mlp(m, p, i)
     xf = _ln(X, p, "lnf")
@@ -59,8 +64,8 @@ def model_loss(params, variant, heads, tokens, targets, layers, parallel=False):
     return Fn.cross_entropy(logits.reshape(B * T, -1), torch.as_tensor(targets, dtype=torch.long).reshape(-1))
 
 
-def loss_and_grads(params_np, variant, heads, tokens, targets, layers, parallel=False):
+def loss_and_grads(params_np, variant, heads, tokens, targets, layers, parallel=False, **kw):
     p = {k: torch.tensor(v, dtype=torch.float64, requires_grad=True) for k, v in params_np.items()}
-    loss = model_loss(p, variant, heads, tokens, targets, layers, parallel)
+    loss = model_loss(p, variant, heads, tokens, targets, layers, parallel, **kw)
     loss.backward()
     return float(loss), {k: t.grad.numpy() if t.grad is not None else torch.zeros_like(t).numpy() for k, t in p.items()}
