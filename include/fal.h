@@ -9,6 +9,12 @@
  *        LayerNorm shared by all blocks (applied "only once", Sec. 4.1).
  *   FAL+ (Sec. 5, App. D.1): block 1 is the standard block; block i >= 2 feeds
  *        MLP_i(LN(X_i + MHA_i(LN(X_i))) + LN_{F,i}(MHA_1(LN(X_1)))).
+ * The paper's comparison blocks, built from the same kernels:
+ *   Parallel (Sec. 5.1, GPT-J style): X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i)).
+ *   Ablation1 (App. D): X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i) + LN_{A,i}(MHA_i(LN(X_i)))).
+ *   Ablation2 (App. D): block 1 standard, every later block Parallel.
+ *   FAL+ reusing block k (App. D, "Ablation with Other Layers"): blocks 1..k
+ *        standard, block i > k adds LN_{F,i}(MHA_k(LN(X_k))) (reuse_layer = k).
  * GPT-2 conventions: learned positions, tied LM head, final LN, biases on every
  * linear map, tanh GELU, LN eps 1e-5, causal attention scaled by 1/sqrt(head_dim),
  * mean token cross-entropy; AdamW with bias correction and decoupled weight
@@ -46,6 +52,9 @@ extern "C" {
 #define FAL_GPT 0
 #define FAL_FAL 1
 #define FAL_FALPLUS 2
+#define FAL_PARALLEL 3
+#define FAL_ABLATION1 4
+#define FAL_ABLATION2 5
 
 /* arithmetic of the path */
 #define FAL_BF16 0        /* bf16 tensor-core GEMMs/attention, fp32 accumulation, fp32 residual */
@@ -56,7 +65,7 @@ extern "C" {
 #define FAL_SCHED_TWO_STREAM 1  /* FAL blocks i >= 2: MHA branch on stream_side, MLP on stream_main */
 
 typedef struct fal_config {
-    int variant;      /* FAL_GPT | FAL_FAL | FAL_FALPLUS */
+    int variant;      /* FAL_GPT | FAL_FAL | FAL_FALPLUS | FAL_PARALLEL | FAL_ABLATION1 | FAL_ABLATION2 */
     int layers;       /* L >= 1 */
     int d_model;      /* d, multiple of 8 (bf16) or 4 (fp32 debug) */
     int heads;        /* H, d % H == 0; bf16 needs head_dim in {64, 128} */
@@ -67,10 +76,19 @@ typedef struct fal_config {
     int precision;    /* FAL_BF16 | FAL_FP32_DEBUG */
     int schedule;     /* FAL_SCHED_* */
     float lr, beta1, beta2, eps, weight_decay;  /* AdamW */
+    int reuse_layer;  /* FAL+ only: block k (1-based) whose attention output later blocks add;
+                         0 or 1 = the first block (FAL+ as defined); other variants need 0 or 1 */
+    float clip_norm;  /* > 0: before AdamW, scale the gradients so that their global L2 norm is
+                         at most clip_norm (App. A clips at 1.0); 0 = no clipping.  With
+                         clipping, fal_train_step cannot update weights inside the gradient
+                         GEMMs (the norm needs every gradient first) and runs AdamW after
+                         the backward, like fal_step. */
 } fal_config;
 
 typedef struct fal_tensor_info {
-    char name[48];   /* e.g. "wte", "h3.attn.w_qkv", "lnF.g" (layers numbered from 0) */
+    char name[48];   /* e.g. "wte", "h3.attn.w_qkv", "lnF.g" (layers numbered from 0); per-block
+                        LayerNorms: ln1, ln2 (GPT-style MLP input), lnF (FAL+ first-attention
+                        term), lnA (Ablation1 own-attention term) */
     size_t offset;   /* first element inside the flat fp32 parameter buffer */
     size_t numel;
     int ndim;        /* 1 or 2 */
@@ -111,6 +129,11 @@ int fal_step(fal_handle* h);
 
 /* forward + backward + step. */
 int fal_train_step(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host);
+
+/* Global L2 norm of the gradients before clipping, as computed by the last
+ * fal_step / fal_train_step with clip_norm > 0 (synchronizes).  FAL_ERR_STATE
+ * if no clipped step ran yet. */
+int fal_get_grad_norm(fal_handle* h, float* norm_host);
 
 /* Waits for both streams and reports device-side errors (token range, wait timeouts). */
 int fal_sync(fal_handle* h);

@@ -420,17 +420,65 @@ __global__ void add_scaled_cols_kernel(long n, int d, const float* __restrict__ 
 // shadow (bf16 copy of p) refreshed in the same pass.
 __global__ void adamw_kernel(size_t n, size_t n_decay, float* __restrict__ p, const float* __restrict__ g,
                              float* __restrict__ m, float* __restrict__ v, bf16* __restrict__ shadow, float lr,
-                             float b1, float b2, float eps, float wd, float rbc1, float rbc2) {
+                             float b1, float b2, float eps, float wd, float rbc1, float rbc2,
+                             const float* __restrict__ gscale) {
   const size_t n4 = n / 4;
+  const float gs = gscale ? *gscale : 1.f;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
     const size_t e = i * 4;
     float4 pp = load4(p + e), gg = load4(g + e), mm = load4(m + e), vv = load4(v + e);
+    gg.x *= gs; gg.y *= gs; gg.z *= gs; gg.w *= gs;
     float* pa = &pp.x; float* ga = &gg.x; float* ma = &mm.x; float* va = &vv.x;
 #pragma unroll
     for (int j = 0; j < 4; ++j)
       adamw_elem(pa[j], ma[j], va[j], ga[j], lr, b1, b2, eps, (e + j < n_decay) ? wd : 0.f, rbc1, rbc2);
     store4(p + e, pp); store4(m + e, mm); store4(v + e, vv);
     if (shadow) store4(shadow + e, pp);
+  }
+}
+
+// Sum of squares of g over this block's contiguous slice (16-byte loads, fp32
+// per thread, fp64 across threads): one partial per block, in block order.
+constexpr int GN_BLOCKS = 1024, GN_THREADS = 256;
+__global__ void __launch_bounds__(GN_THREADS) grad_sumsq_kernel(size_t n4, const float* __restrict__ g,
+                                                                 double* __restrict__ partial) {
+  const size_t per = (n4 + gridDim.x - 1) / gridDim.x;
+  const size_t b0 = blockIdx.x * per, b1 = b0 + per < n4 ? b0 + per : n4;
+  float acc = 0.f;
+  for (size_t i = b0 + threadIdx.x; i < b1; i += blockDim.x) {
+    const float4 v = load4(g + 4 * i);
+    acc = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, acc))));
+  }
+  double s = acc;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ double sh[GN_THREADS / 32];
+  if (threadIdx.x % 32 == 0) sh[threadIdx.x / 32] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < GN_THREADS / 32; ++w) t += sh[w];
+    partial[blockIdx.x] = t;
+  }
+}
+
+// norm = sqrt(sum of the partials in block order); scale = max_norm / norm when
+// the norm exceeds max_norm, else 1.
+__global__ void grad_clip_finish_kernel(int nb, const double* __restrict__ partial, float max_norm,
+                                        float* __restrict__ norm_out, float* __restrict__ scale_out) {
+  __shared__ double sh[32];
+  double s = 0.0;
+  const int per = (nb + 31) / 32;
+  if (threadIdx.x < 32)
+    for (int b = threadIdx.x * per; b < (threadIdx.x + 1) * per && b < nb; ++b) s += partial[b];
+  if (threadIdx.x < 32) sh[threadIdx.x] = s;
+  __syncwarp();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 32; ++w) t += sh[w];
+    const double norm = sqrt(t);
+    *norm_out = (float)norm;
+    *scale_out = norm > (double)max_norm ? (float)((double)max_norm / norm) : 1.f;
   }
 }
 
@@ -606,13 +654,25 @@ int add_scaled_cols(int rows, int d, const float* src, const float* colvec, floa
 }
 
 int adamw(size_t n, size_t n_decay, float* p, const float* g, float* m, float* v, void* shadow, float lr, float beta1,
-          float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s) {
+          float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s, const float* gscale) {
   if (n == 0) return 0;
   if (n % 4) return 1;
   const int blocks = num_sms() * 8;
   adamw_kernel<<<blocks, 256, 0, s>>>(n, n_decay, p, g, m, v, reinterpret_cast<bf16*>(shadow), lr, beta1, beta2, eps, wd,
-                                      1.f / bc1, 1.f / bc2);
+                                      1.f / bc1, 1.f / bc2, gscale);
   count_launches(1);
+  return last_err();
+}
+
+int grad_norm_partials() { return 2 * GN_BLOCKS; }  // GN_BLOCKS doubles
+
+int grad_norm_clip(size_t n, const float* g, float max_norm, float* partial, float* norm_out, float* scale_out,
+                   cudaStream_t s) {
+  if (n % 4) return 1;
+  double* part = reinterpret_cast<double*>(partial);
+  grad_sumsq_kernel<<<GN_BLOCKS, GN_THREADS, 0, s>>>(n / 4, g, part);
+  grad_clip_finish_kernel<<<1, 32, 0, s>>>(GN_BLOCKS, part, max_norm, norm_out, scale_out);
+  count_launches(2);
   return last_err();
 }
 

@@ -142,8 +142,17 @@ int cross_entropy(int act_bf16, int rows, int V, long ld, const void* logits, co
                   void* dlogits, float* loss_rows, float* loss, int* err, cudaStream_t s);
 // dst += src * colvec (per column), fp32 [rows, d]
 int add_scaled_cols(int rows, int d, const float* src, const float* colvec, float* dst, cudaStream_t s);
+// gscale: device scalar multiplying every gradient (gradient clipping), or null.
 int adamw(size_t n, size_t n_decay, float* p, const float* g, float* m, float* v, void* shadow_bf16,
-          float lr, float beta1, float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s);
+          float lr, float beta1, float beta2, float eps, float wd, float bc1, float bc2, cudaStream_t s,
+          const float* gscale = nullptr);
+// Global L2 norm of g[0..n) (n a multiple of 4) and the clipping factor
+// min(1, max_norm / norm), both written to device scalars; deterministic
+// (fixed per-block partials summed in a fixed order).  partial: scratch of
+// grad_norm_partials() floats.
+int grad_norm_clip(size_t n, const float* g, float max_norm, float* partial, float* norm_out, float* scale_out,
+                   cudaStream_t s);
+int grad_norm_partials();
 int f32_to_bf16(size_t n, const float* src, void* dst, cudaStream_t s);
 int act_to_f32(int act_bf16, size_t n, const void* src, float* dst, cudaStream_t s);
 // copy [rows, cols] from a strided activation into dense fp32

@@ -1,5 +1,7 @@
 // Runtime behind the C ABI: workspace layout, the forward/backward schedule of
-// GPT (Eq. 1), FAL (Eq. 2) and FAL+ (App. D.1) decoder stacks, AdamW, taps.
+// GPT (Eq. 1), FAL (Eq. 2) and FAL+ (App. D.1) decoder stacks and of the
+// paper's comparison blocks (Parallel, Sec. 5.1; Ablation1 / Ablation2 and FAL+
+// reusing block k, App. D), AdamW with optional gradient clipping, taps.
 //
 // Data layout (all carved from the caller's workspace, 256-byte aligned):
 //   flat fp32 parameters / gradients / AdamW m, v   [n_params]
@@ -33,7 +35,7 @@ constexpr size_t NPOS = (size_t)-1;
 
 struct LayerP {
   size_t ln1_g = NPOS, ln1_b = NPOS, w_qkv = NPOS, b_qkv = NPOS, w_o = NPOS, b_o = NPOS;
-  size_t ln2_g = NPOS, ln2_b = NPOS, lnF_g = NPOS, lnF_b = NPOS;
+  size_t ln2_g = NPOS, ln2_b = NPOS, lnF_g = NPOS, lnF_b = NPOS, lnA_g = NPOS, lnA_b = NPOS;
   size_t w_up = NPOS, b_up = NPOS, w_down = NPOS, b_down = NPOS;
 };
 
@@ -43,6 +45,16 @@ struct LayerA {
   void *u = nullptr, *m = nullptr, *qkv = nullptr, *ctx = nullptr, *h = nullptr, *g = nullptr;
   float* lse = nullptr;
   float *Y = nullptr, *ln2_mean = nullptr, *ln2_rstd = nullptr;
+  // Ablation1: the block's own attention output a_i and its normalised form
+  float *a = nullptr, *ahat = nullptr, *a_mean = nullptr, *a_rstd = nullptr;
+};
+
+// How block i computes its MLP input.
+enum BlockKind {
+  BK_SEQ = 0,     // m = LN2(X + a) (+ LN_{F,i}(a_k) for FAL+ after block k): GPT-style, sequential
+  BK_PAR = 1,     // m = LN1(X) (+ LN_F(a_1) for FAL): the branches run side by side (Eq. 2)
+  BK_FIRST = 2,   // FAL block 1: m = LN1(X) + LN_F(a_1) with a_1 computed here
+  BK_OWN = 3      // Ablation1: m = LN1(X) + LN_{A,i}(a_i), the block's own attention
 };
 
 struct Bump {
@@ -106,6 +118,10 @@ struct fal_handle {
   float *dX = nullptr, *dY = nullptr, *dA = nullptr, *dU = nullptr, *dU2 = nullptr, *dA1hat = nullptr;
   void *dX_act = nullptr, *dY_act = nullptr, *dA_act = nullptr, *dctx = nullptr, *dh = nullptr, *dqkv = nullptr;
   float *dvec = nullptr, *part0 = nullptr, *part1 = nullptr;
+  // gradient clipping: per-block partials, the norm and the scale factor
+  float *gn_part = nullptr, *gn_norm = nullptr, *gn_scale = nullptr;
+  bool has_norm = false;
+  int reuse = 0;  // 0-based block whose attention output FAL+ adds to later MLP inputs
   float* stage = nullptr;
   size_t stage_floats = 0;
   size_t total_bytes = 0;
@@ -154,13 +170,17 @@ void build_table(fal_handle* h) {
     add_tensor(h, dec, nodec, p + "attn.b_qkv", 3 * d, 0, 0);
     add_tensor(h, dec, nodec, p + "attn.w_o", d, d, 1);
     add_tensor(h, dec, nodec, p + "attn.b_o", d, 0, 0);
-    if (var == FAL_GPT || var == FAL_FALPLUS) {
+    if (var == FAL_GPT || var == FAL_FALPLUS || (var == FAL_ABLATION2 && i == 0)) {
       add_tensor(h, dec, nodec, p + "ln2.g", d, 0, 0);
       add_tensor(h, dec, nodec, p + "ln2.b", d, 0, 0);
     }
-    if (var == FAL_FALPLUS && i >= 1) {
+    if (var == FAL_FALPLUS && i > h->reuse) {
       add_tensor(h, dec, nodec, p + "lnF.g", d, 0, 0);
       add_tensor(h, dec, nodec, p + "lnF.b", d, 0, 0);
+    }
+    if (var == FAL_ABLATION1) {
+      add_tensor(h, dec, nodec, p + "lnA.g", d, 0, 0);
+      add_tensor(h, dec, nodec, p + "lnA.b", d, 0, 0);
     }
     add_tensor(h, dec, nodec, p + "mlp.w_up", F, d, 1);
     add_tensor(h, dec, nodec, p + "mlp.b_up", F, 0, 0);
@@ -211,6 +231,8 @@ void build_table(fal_handle* h) {
       else if (leaf == "ln2.b") q.ln2_b = t.offset;
       else if (leaf == "lnF.g") q.lnF_g = t.offset;
       else if (leaf == "lnF.b") q.lnF_b = t.offset;
+      else if (leaf == "lnA.g") q.lnA_g = t.offset;
+      else if (leaf == "lnA.b") q.lnA_b = t.offset;
       else if (leaf == "mlp.w_up") q.w_up = t.offset;
       else if (leaf == "mlp.b_up") q.b_up = t.offset;
       else if (leaf == "mlp.w_down") q.w_down = t.offset;
@@ -221,12 +243,20 @@ void build_table(fal_handle* h) {
 
 int validate(const fal_config* c, std::string* msg) {
   if (!c) { *msg = "null config"; return FAL_ERR_ARG; }
-  if (c->variant < FAL_GPT || c->variant > FAL_FALPLUS) { *msg = "variant must be GPT, FAL or FAL+"; return FAL_ERR_ARG; }
+  if (c->variant < FAL_GPT || c->variant > FAL_ABLATION2) {
+    *msg = "variant must be GPT, FAL, FAL+, Parallel, Ablation1 or Ablation2";
+    return FAL_ERR_ARG;
+  }
   if (c->layers < 1 || c->d_model < 1 || c->heads < 1 || c->d_ff < 1 || c->seq < 1 || c->batch < 1 || c->vocab < 2) {
     *msg = "layers, d_model, heads, d_ff, seq, batch must be >= 1 and vocab >= 2";
     return FAL_ERR_ARG;
   }
   if (c->d_model % c->heads) { *msg = "d_model must be a multiple of heads"; return FAL_ERR_ARG; }
+  if (c->reuse_layer < 0 || c->reuse_layer > c->layers || (c->reuse_layer > 1 && c->variant != FAL_FALPLUS)) {
+    *msg = "reuse_layer must be in [0, layers] and above 1 only for FAL+";
+    return FAL_ERR_ARG;
+  }
+  if (!(c->clip_norm >= 0.f)) { *msg = "clip_norm must be >= 0"; return FAL_ERR_ARG; }
   if (c->precision != FAL_BF16 && c->precision != FAL_FP32_DEBUG) { *msg = "bad precision"; return FAL_ERR_ARG; }
   if (c->schedule != FAL_SCHED_SERIAL && c->schedule != FAL_SCHED_TWO_STREAM) { *msg = "bad schedule"; return FAL_ERR_ARG; }
   const int hd = c->d_model / c->heads;
@@ -250,6 +280,23 @@ void init_dims(fal_handle* h, const fal_config* c) {
   h->F = c->d_ff; h->L = c->layers; h->V = c->vocab;
   h->Vp = (c->vocab + 63) / 64 * 64;
   h->BT = (long)h->B * h->T;
+  h->reuse = c->reuse_layer > 1 ? c->reuse_layer - 1 : 0;
+}
+
+// MLP-input rule of block i (the block equations of each variant).
+int block_kind(const fal_handle* h, int i) {
+  switch (h->cfg.variant) {
+    case FAL_FAL: return i == 0 ? BK_FIRST : BK_PAR;
+    case FAL_PARALLEL: return BK_PAR;
+    case FAL_ABLATION1: return BK_OWN;
+    case FAL_ABLATION2: return i == 0 ? BK_SEQ : BK_PAR;
+    default: return BK_SEQ;  // GPT, FAL+
+  }
+}
+// The tensor the MLP reads: m, or u itself where the MLP input is LN1(X) alone.
+const void* mlp_in(const fal_handle* h, int i) {
+  const int v = h->cfg.variant;
+  return (block_kind(h, i) == BK_PAR && v != FAL_FAL) ? h->la[i].u : h->la[i].m;
 }
 
 // Carves every buffer; with base == nullptr it only measures.
@@ -284,10 +331,16 @@ void carve(fal_handle* h, uint8_t* base) {
     A.lse = b.take<float>((size_t)h->B * h->H * h->T);
     A.h = b.take<uint8_t>(BT * F * a);
     A.g = b.take<uint8_t>(BT * F * a);
-    if (var != FAL_FAL) {
+    if (var == FAL_GPT || var == FAL_FALPLUS || (var == FAL_ABLATION2 && i == 0)) {
       A.Y = b.take<float>(BT * d);
       A.ln2_mean = b.take<float>(BT);
       A.ln2_rstd = b.take<float>(BT);
+    }
+    if (var == FAL_ABLATION1) {
+      A.a = b.take<float>(BT * d);
+      A.ahat = b.take<float>(BT * d);
+      A.a_mean = b.take<float>(BT);
+      A.a_rstd = b.take<float>(BT);
     }
   }
   h->Xout = b.take<float>(BT * d);
@@ -316,6 +369,9 @@ void carve(fal_handle* h, uint8_t* base) {
   const int cs_cols = 3 * h->d > h->F ? 3 * h->d : h->F;  // widest column reduction: b_qkv or b_up
   h->part0 = b.take<float>(colsum_partial_floats(cs_cols));
   h->part1 = b.take<float>(colsum_partial_floats(cs_cols));
+  h->gn_part = b.take<float>(grad_norm_partials());
+  h->gn_norm = b.take<float>(4);
+  h->gn_scale = b.take<float>(4);
   h->stage_floats = (size_t)4 << 20;
   h->stage = b.take<float>(h->stage_floats);
   h->total_bytes = b.off + ALIGN;
@@ -511,7 +567,8 @@ void up_gemm(Ctx& c, int i, cudaStream_t s) {
   const LayerP& p = h->lp[i];
   EpiParams e = epi_out(A.h, h->F, OUT_ACT);
   e.op = EPI_GELU; e.out2 = A.g; e.ldo2 = h->F; e.bias = Pp(h, p.b_up);
-  gemm(c, call1((int)h->BT, h->F, seg(A.m, h->d, 0, Wp(h, p.w_up), h->d, 0, h->d), e), s, "MLP up-projection");
+  gemm(c, call1((int)h->BT, h->F, seg(mlp_in(h, i), h->d, 0, Wp(h, p.w_up), h->d, 0, h->d), e), s,
+       "MLP up-projection");
 }
 
 // Whether splitting an M x N output of 256 x 256 tiles (one per pair of SMs)
@@ -529,10 +586,14 @@ void layer_forward(Ctx& c, int i) {
   const int BT = (int)h->BT, d = h->d, F = h->F, var = h->cfg.variant;
   float* Xn = (i + 1 < h->L) ? h->la[i + 1].X : h->Xout;
   cudaStream_t s = h->sm;
-  if (var == FAL_FAL && i >= 1) {
-    // m_i = LN1_i(X_i) + a1hat * gamma_F + beta_F  (Eq. 2), u_i = LN1_i(X_i)
-    ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), A.u, nullptr, A.ln1_mean, A.ln1_rstd, A.m, h->a1hat,
-            Pp(h, h->lnF_g), Pp(h, h->lnF_b));
+  const int kind = block_kind(h, i);
+  if (kind == BK_PAR) {
+    if (var == FAL_FAL)  // m_i = LN1_i(X_i) + a1hat * gamma_F + beta_F  (Eq. 2), u_i = LN1_i(X_i)
+      ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), A.u, nullptr, A.ln1_mean, A.ln1_rstd, A.m, h->a1hat,
+              Pp(h, h->lnF_g), Pp(h, h->lnF_b));
+    else  // Parallel block: the MLP reads u_i = LN1_i(X_i) itself
+      ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), A.u, nullptr, A.ln1_mean, A.ln1_rstd, nullptr, nullptr,
+              nullptr, nullptr);
     // The MHA branch and the MLP branch only share u/m: run them side by side.
     const bool two = h->cfg.schedule == FAL_SCHED_TWO_STREAM && h->ss != h->sm;
     if (two) {
@@ -581,31 +642,37 @@ void layer_forward(Ctx& c, int i) {
   ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), A.u, nullptr, A.ln1_mean, A.ln1_rstd, nullptr, nullptr, nullptr,
           nullptr);
   qkv_and_attention(c, i, s);
-  if (var == FAL_FAL) {
-    // block 1 of FAL: a_1 = ctx W_o^T + b_o, a1hat = LN(a_1) without affine,
-    // m_1 = LN1_1(X_1) + F, X_2 = X_1 + a_1 + MLP_1(m_1)
-    EpiParams e = epi_out(h->a1, d, OUT_F32);
+  if (kind == BK_FIRST || kind == BK_OWN) {
+    // FAL block 1: a_1 = ctx W_o^T + b_o, a1hat = LN(a_1) without affine,
+    // m_1 = LN1_1(X_1) + a1hat * gamma_F + beta_F, X_2 = X_1 + a_1 + MLP_1(m_1).
+    // Ablation1 block i: the same with the block's own a_i and LN_{A,i}.
+    const bool first = kind == BK_FIRST;
+    float* a = first ? h->a1 : A.a;
+    float* ahat = first ? h->a1hat : A.ahat;
+    EpiParams e = epi_out(a, d, OUT_F32);
     e.bias = Pp(h, p.b_o);
     gemm(c, call1(BT, d, seg(A.ctx, d, 0, Wp(h, p.w_o), d, 0, d), e), s, "attention output projection");
-    ln_fwd_(c, s, h->a1, nullptr, nullptr, nullptr, h->a1hat, h->a1_mean, h->a1_rstd, nullptr, nullptr, nullptr,
-            nullptr);
-    ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), nullptr, nullptr, nullptr, nullptr, A.m, h->a1hat,
-            Pp(h, h->lnF_g), Pp(h, h->lnF_b));
+    ln_fwd_(c, s, a, nullptr, nullptr, nullptr, ahat, first ? h->a1_mean : A.a_mean, first ? h->a1_rstd : A.a_rstd,
+            nullptr, nullptr, nullptr, nullptr);
+    ln_fwd_(c, s, A.X, Pp(h, p.ln1_g), Pp(h, p.ln1_b), nullptr, nullptr, nullptr, nullptr, A.m, ahat,
+            Pp(h, first ? h->lnF_g : p.lnA_g), Pp(h, first ? h->lnF_b : p.lnA_b));
     up_gemm(c, i, s);
     EpiParams e2 = epi_out(Xn, d, OUT_F32);
-    e2.bias = Pp(h, p.b_down); e2.resid = A.X; e2.ldr = d; e2.resid2 = h->a1; e2.ldr2 = d;
+    e2.bias = Pp(h, p.b_down); e2.resid = A.X; e2.ldr = d; e2.resid2 = a; e2.ldr2 = d;
     gemm(c, call1(BT, d, seg(A.g, F, 0, Wp(h, p.w_down), F, 0, F), e2), s, "MLP down-projection");
     return;
   }
-  // GPT and FAL+: Y = X + a; m = LN2(Y) (+ LN_{F,i}(a_1) for FAL+ i >= 2)
+  // GPT, FAL+ and Ablation2's block 1: Y = X + a; m = LN2(Y) (+ LN_{F,i}(a_k)
+  // for FAL+ blocks after the reused block k)
+  const bool keep_a = var == FAL_FALPLUS && i == h->reuse;
   EpiParams e = epi_out(A.Y, d, OUT_F32);
   e.bias = Pp(h, p.b_o); e.resid = A.X; e.ldr = d;
-  if (var == FAL_FALPLUS && i == 0) { e.pre_f32 = 1; e.out2 = h->a1; e.ldo2 = d; }
+  if (keep_a) { e.pre_f32 = 1; e.out2 = h->a1; e.ldo2 = d; }
   gemm(c, call1(BT, d, seg(A.ctx, d, 0, Wp(h, p.w_o), d, 0, d), e), s, "attention output projection");
-  if (var == FAL_FALPLUS && i == 0)
+  if (keep_a)
     ln_fwd_(c, s, h->a1, nullptr, nullptr, nullptr, h->a1hat, h->a1_mean, h->a1_rstd, nullptr, nullptr, nullptr,
             nullptr);
-  if (var == FAL_FALPLUS && i >= 1)
+  if (var == FAL_FALPLUS && i > h->reuse)
     ln_fwd_(c, s, A.Y, Pp(h, p.ln2_g), Pp(h, p.ln2_b), nullptr, nullptr, A.ln2_mean, A.ln2_rstd, A.m, h->a1hat,
             Pp(h, p.lnF_g), Pp(h, p.lnF_b));
   else
@@ -662,7 +729,7 @@ void mlp_backward(Ctx& c, int i, const float* dXn, const void* dXn_act, cudaStre
                        call1(BT, F, dgrad_seg(h, dXn_act, d, p.w_down, F), e)}),
        s, "MLP down wgrad + dgrad");
   colsum_(c, s, part, dXn, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_down), nullptr, 0);
-  gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), wgrad_out(h, p.w_up, d)),
+  gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, mlp_in(h, i), d), wgrad_out(h, p.w_up, d)),
                        call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
        s, "MLP up wgrad + dgrad");
   colsum_(c, s, part, h->dh, 1, F, F, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_up), nullptr, 0);
@@ -702,16 +769,18 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
           nullptr, 0);
 }
 
-// first-attention term of MLP_i's input: dA1hat += dU2 * gamma_F(i); dgamma_F(i), dbeta_F(i)
-void first_attention_grad(Ctx& c, size_t g_off, size_t b_off, cudaStream_t s, float* part, int accumulate) {
+// attention term of MLP_i's input (first attention, or Ablation1's own):
+// dA1hat += dU2 * gamma(i); dgamma(i), dbeta(i) from the normalised ahat
+void first_attention_grad(Ctx& c, size_t g_off, size_t b_off, cudaStream_t s, float* part, int accumulate,
+                          const float* ahat = nullptr) {
   fal_handle* h = c.h;
   if (!c.ok()) return;
   {
     ProfScope ps(h, s, 3, 0.0, "first-attention gradient");
     c.check(add_scaled_cols((int)h->BT, h->d, h->dU2, Pp(h, g_off), h->dA1hat, s), "first-attention gradient");
   }
-  colsum_(c, s, part, h->dU2, 0, h->d, h->d, nullptr, 2, nullptr, nullptr, nullptr, h->a1hat, Gp(h, g_off), Gp(h, b_off),
-          nullptr, accumulate);
+  colsum_(c, s, part, h->dU2, 0, h->d, h->d, nullptr, 2, nullptr, nullptr, nullptr, ahat ? ahat : h->a1hat,
+          Gp(h, g_off), Gp(h, b_off), nullptr, accumulate);
 }
 
 void layer_backward(Ctx& c, int i) {
@@ -721,7 +790,8 @@ void layer_backward(Ctx& c, int i) {
   const int BT = (int)h->BT, d = h->d, F = h->F, var = h->cfg.variant;
   cudaStream_t s = h->sm;
   // dX / dX_act hold the gradient w.r.t. X_{i+1} on entry and X_i on exit.
-  if (var == FAL_FAL && i >= 1) {
+  const int kind = block_kind(h, i);
+  if (kind == BK_PAR) {
     // One launch for the fused residual GEMM's gradients:
     // [dW_o | dW_down] = dX^T [ctx | g] and [dctx | dh] = dX [W_o | W_down] (dh with gelu').
     EpiParams edh = epi_out(h->dh, F, OUT_ACT);
@@ -742,22 +812,29 @@ void layer_backward(Ctx& c, int i) {
     cudaStream_t sa = two ? h->ss : s;
     if (two) fork(h);
     attn_backward(c, i, nullptr, nullptr, sa, two ? h->part1 : h->part0, true, h->bf != 0);
-    gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, A.m, d), wgrad_out(h, p.w_up, d)),
+    gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, mlp_in(h, i), d), wgrad_out(h, p.w_up, d)),
                          call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
          s, "MLP up wgrad + dgrad");
     colsum_(c, s, h->part0, h->dh, 1, F, F, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_up),
             nullptr, 0);
-    first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
+    if (var == FAL_FAL) first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
     if (two) join(h);
     ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
             h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
     return;
   }
-  if (var == FAL_FAL) {  // block 1
+  if (kind == BK_FIRST || kind == BK_OWN) {  // FAL block 1, Ablation1 blocks
+    const bool first = kind == BK_FIRST;
     mlp_backward(c, i, h->dX, h->dX_act, s, h->part0);
-    first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
-    // da_1 = dX_2 + (LN without affine)'(a_1) . dA1hat   (a_1 feeds X_2 and F)
-    ln_bwd_(c, s, h->dA1hat, nullptr, h->a1, h->a1_mean, h->a1_rstd, nullptr, h->dX, h->dA, h->dA_act);
+    if (first) {
+      first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
+    } else {
+      cudaMemsetAsync(h->dA1hat, 0, (size_t)BT * d * 4, s);
+      first_attention_grad(c, p.lnA_g, p.lnA_b, s, h->part0, 0, A.ahat);
+    }
+    // da = dX_{i+1} + (LN without affine)'(a) . dA1hat   (a feeds X_{i+1} and the MLP input)
+    ln_bwd_(c, s, h->dA1hat, nullptr, first ? h->a1 : A.a, first ? h->a1_mean : A.a_mean,
+            first ? h->a1_rstd : A.a_rstd, nullptr, h->dX, h->dA, h->dA_act);
     attn_backward(c, i, h->dA, h->dA_act, s, h->part0, false);
     ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
             h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
@@ -769,8 +846,8 @@ void layer_backward(Ctx& c, int i) {
           h->part0, Gp(h, p.ln2_g), Gp(h, p.ln2_b));
   const float* da = h->dY;
   const void* da_act = h->dY_act;
-  if (var == FAL_FALPLUS && i >= 1) first_attention_grad(c, p.lnF_g, p.lnF_b, s, h->part0, 0);
-  if (var == FAL_FALPLUS && i == 0) {
+  if (var == FAL_FALPLUS && i > h->reuse) first_attention_grad(c, p.lnF_g, p.lnF_b, s, h->part0, 0);
+  if (var == FAL_FALPLUS && i == h->reuse) {
     ln_bwd_(c, s, h->dA1hat, nullptr, h->a1, h->a1_mean, h->a1_rstd, nullptr, h->dY, h->dA, h->dA_act);
     da = h->dA;
     da_act = h->dA_act;
@@ -891,6 +968,16 @@ void fal_destroy(fal_handle* h) {
   delete h;
 }
 
+int fal_get_grad_norm(fal_handle* h, float* norm_host) {
+  if (!h || !norm_host) return FAL_ERR_ARG;
+  if (!h->has_norm) return fail(h, FAL_ERR_STATE, "no step with gradient clipping yet");
+  int r = read_dev_err(h);
+  if (r) return r;
+  if (cudaMemcpy(norm_host, h->gn_norm, sizeof(float), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return fail(h, FAL_ERR_CUDA, "norm copy failed");
+  return FAL_OK;
+}
+
 int fal_sync(fal_handle* h) {
   if (!h) return FAL_ERR_ARG;
   return read_dev_err(h);
@@ -938,7 +1025,18 @@ int adamw_range(fal_handle* h, size_t begin, size_t end, size_t decay_end) {
   const float bc2 = 1.f - (float)pow((double)c.beta2, (double)h->step_t);
   void* sh = h->bf ? (void*)((uint8_t*)h->Shb[h->sh_cur ^ 1] + begin * 2) : nullptr;
   return adamw(end - begin, decay_end > begin ? decay_end - begin : 0, h->P + begin, h->G + begin, h->Mo + begin,
-               h->Vo + begin, sh, c.lr, c.beta1, c.beta2, c.eps, c.weight_decay, bc1, bc2, h->sm);
+               h->Vo + begin, sh, c.lr, c.beta1, c.beta2, c.eps, c.weight_decay, bc1, bc2, h->sm,
+               h->cfg.clip_norm > 0.f ? h->gn_scale : nullptr);
+}
+
+// Gradient clipping (App. A): the global norm of the whole flat gradient
+// buffer (its padding is zero) and the factor AdamW applies to every gradient.
+int clip_grads(fal_handle* h) {
+  if (h->cfg.clip_norm <= 0.f) return 0;
+  ProfScope ps(h, h->sm, 3, 0.0, "gradient norm");
+  const int r = grad_norm_clip(h->n_params, h->G, h->cfg.clip_norm, h->gn_part, h->gn_norm, h->gn_scale, h->sm);
+  if (r == 0) h->has_norm = true;
+  return r;
 }
 }  // namespace
 
@@ -946,6 +1044,7 @@ int fal_step(fal_handle* h) {
   if (!h) return FAL_ERR_ARG;
   if (h->state < 2) return fail(h, FAL_ERR_STATE, "fal_step needs a preceding fal_backward");
   h->step_t += 1;
+  if (clip_grads(h)) return fail(h, FAL_ERR_CUDA, "gradient norm launch failed");
   if (adamw_range(h, 0, h->n_params, h->n_decay)) return fail(h, FAL_ERR_CUDA, "AdamW launch failed");
   h->sh_cur ^= 1;
   h->state = 0;
@@ -965,12 +1064,14 @@ int fal_train_step(fal_handle* h, const int32_t* tokens, const int32_t* targets,
     h->opt_rbc2 = 1.f / (1.f - (float)pow((double)c.beta2, (double)h->step_t));
   }
   // (bf16 path only: the fp32 debug path's GEMMs read the fp32 master weights,
-  // which the fused update would overwrite under a concurrent reader.)
-  const bool fused = h->bf != 0;
+  // which the fused update would overwrite under a concurrent reader.  With
+  // gradient clipping the update needs the norm of every gradient first.)
+  const bool fused = h->bf != 0 && !(h->cfg.clip_norm > 0.f);
   h->fuse_opt = fused;
   r = backward_impl(h);
   h->fuse_opt = false;
   if (r) return r;
+  if (clip_grads(h)) return fail(h, FAL_ERR_CUDA, "gradient norm launch failed");
   const size_t blocks_begin = h->lp[0].w_qkv;
   const bool bad = fused ? (adamw_range(h, 0, blocks_begin, blocks_begin) ||
                             adamw_range(h, h->n_decay, h->n_params, h->n_decay))
@@ -1070,7 +1171,7 @@ int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n
     is_act = 0;
   } else if (nm == "Y") { if (lay) src = h->la[layer].Y; is_act = 0; }
   else if (nm == "u") { if (lay) src = h->la[layer].u; }
-  else if (nm == "m") { if (lay) src = h->la[layer].m; }
+  else if (nm == "m") { if (lay) src = mlp_in(h, layer); }
   else if (nm == "ctx") { if (lay) src = h->la[layer].ctx; }
   else if (nm == "qkv") { if (lay) src = h->la[layer].qkv; cols = 3 * d; ld = 3L * d; }
   else if (nm == "h") { if (lay) src = h->la[layer].h; cols = F; ld = F; }

@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libfal.so")
 
 FAL_OK, FAL_ERR_ARG, FAL_ERR_STATE, FAL_ERR_WORKSPACE, FAL_ERR_CUDA, FAL_ERR_TIMEOUT, FAL_ERR_UNSUPPORTED = range(7)
-VARIANT = {"gpt": 0, "fal": 1, "falplus": 2}
+VARIANT = {"gpt": 0, "fal": 1, "falplus": 2, "parallel": 3, "ablation1": 4, "ablation2": 5}
 PRECISION = {"bf16": 0, "fp32": 1}
 SCHEDULE = {"serial": 0, "two_stream": 1}
 ENGINE = {"tcgen05": 0, "simt": 1, "tcgen05_pair": 2}
@@ -25,7 +25,8 @@ ENGINE = {"tcgen05": 0, "simt": 1, "tcgen05_pair": 2}
 class FalConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("variant", "layers", "d_model", "heads", "d_ff", "seq", "batch", "vocab",
                                             "precision", "schedule")] + \
-               [(n, ctypes.c_float) for n in ("lr", "beta1", "beta2", "eps", "weight_decay")]
+               [(n, ctypes.c_float) for n in ("lr", "beta1", "beta2", "eps", "weight_decay")] + \
+               [("reuse_layer", ctypes.c_int), ("clip_norm", ctypes.c_float)]
 
 
 class FalTensorInfo(ctypes.Structure):
@@ -61,6 +62,7 @@ _SIGS = {
     "fal_step": (ctypes.c_int, [ctypes.c_void_p]),
     "fal_train_step": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "fal_sync": (ctypes.c_int, [ctypes.c_void_p]),
+    "fal_get_grad_norm": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "fal_get_loss": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "fal_param_count": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_size_t)]),
     "fal_param_info": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int, ctypes.POINTER(FalTensorInfo)]),
@@ -121,9 +123,9 @@ def _stream_ptr(s):
 
 
 def make_config(variant, layers, d_model, heads, d_ff, seq, batch, vocab, precision="bf16", schedule="serial",
-                lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=1e-3):
+                lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=1e-3, reuse_layer=1, clip_norm=0.0):
     return FalConfig(VARIANT[variant], layers, d_model, heads, d_ff, seq, batch, vocab, PRECISION[precision],
-                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay)
+                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay, reuse_layer, clip_norm)
 
 
 def workspace_size(cfg: FalConfig) -> int:
@@ -254,6 +256,11 @@ class Model:
 
     def sync(self):
         _check(lib().fal_sync(self.h), self.h, "fal_sync")
+
+    def grad_norm(self):
+        v = ctypes.c_float()
+        _check(lib().fal_get_grad_norm(self.h, ctypes.byref(v)), self.h, "fal_get_grad_norm")
+        return v.value
 
     def loss(self):
         v = ctypes.c_float()

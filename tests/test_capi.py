@@ -56,6 +56,10 @@ def _ws(cfg):
     dict(layers=0), dict(vocab=1), dict(batch=0),
     dict(d_ff=100),                       # not a multiple of 8
     dict(d_model=4096, heads=32),         # wider than the LN kernels support
+    dict(variant="falplus", reuse_layer=3),   # reuses a block the 2-layer stack does not have
+    dict(reuse_layer=2),                  # reuse_layer applies to FAL+ only
+    dict(clip_norm=-1.0),
+    dict(variant="gpt", layers=-1),
 ])
 def test_workspace_size_rejects_bad_configs(libfal, bad):
     base = dict(variant="fal", layers=2, d_model=128, heads=2, d_ff=512, seq=64, batch=2, vocab=1000)
@@ -66,7 +70,7 @@ def test_workspace_size_rejects_bad_configs(libfal, bad):
 
 def test_workspace_size_accepts_all_shapes(libfal):
     for name, s in synth.SHAPES.items():
-        for v in synth.VARIANTS:
+        for v in synth.ALL_VARIANTS:
             cfg = fal.make_config(v, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
                                   precision=s.precision)
             rc, n = _ws(cfg)
