@@ -198,6 +198,17 @@ int fal_profile_timeline(fal_handle* h, fal_launch_record* out, int cap, int* n)
 /* Number of kernels this library has launched in this process (all handles). */
 long long fal_launch_count(void);
 
+/* Test hook for the library's bounded device waits (the paper has no
+ * counterpart).  With rows >= 0, every CTA of the row-streaming LayerNorm
+ * kernels stops loading rows after `rows` of them, so that the kernel's
+ * waits for the missing rows expire after wait_ns nanoseconds (the default
+ * budget of about one second when wait_ns <= 0); the kernel then records a
+ * timeout and returns, and the next synchronizing call reports
+ * FAL_ERR_TIMEOUT.  rows < 0 restores normal operation (and the default
+ * budget).  Process-wide; for tests only: results computed meanwhile are
+ * invalid. */
+int fal_debug_layernorm_stall(int rows, long long wait_ns);
+
 /* Message for the last failed call on this handle (never NULL). */
 const char* fal_last_error(const fal_handle* h);
 const char* fal_status_string(int status);

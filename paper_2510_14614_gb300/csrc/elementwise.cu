@@ -271,49 +271,54 @@ __global__ void __launch_bounds__(CS_THREADS) colsum_plain_kernel(const src_t* _
   }
 }
 
-// Sums nchunk partials [nchunk][2][d]: slot 0 -> out0 (and out0b), slot 1 -> out1.
-// One CTA per 32 columns: its 8 warps take every 8th chunk (one coalesced
-// 128-byte row segment per warp and slot), then combine through shared memory.
+// Sums nchunk partials [nchunk][NS][d]: slot 0 -> out0 (and out0b), slot 1 ->
+// out1, slot 2 -> out2 (and out2b).  One CTA per 32 columns: its 8 warps take
+// every 8th chunk (one coalesced 128-byte row segment per warp and slot), then
+// combine through shared memory in a fixed order.
 constexpr int CF_WARPS = 8;
+template <int NS>
 __global__ void __launch_bounds__(CF_WARPS * 32) colsum_finish_kernel(const float* __restrict__ partial, int nchunk,
                                                                       int d, float* out1, float* out0, float* out0b,
-                                                                      int accumulate) {
-  __shared__ float red[2][CF_WARPS][32];
+                                                                      float* out2, float* out2b, int accumulate) {
+  __shared__ float red[NS][CF_WARPS][32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x * 32 + lane;
-  float s0 = 0.f, s1 = 0.f;
+  float sv[NS];
+#pragma unroll
+  for (int q = 0; q < NS; ++q) sv[q] = 0.f;
   if (c < d) {
     int k = warp;
     for (; k + 3 * CF_WARPS < nchunk; k += 4 * CF_WARPS) {
-      float a[4], b[4];
+      float a[4][NS];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        a[j] = partial[((long)(k + j * CF_WARPS) * 2 + 0) * d + c];
-        b[j] = partial[((long)(k + j * CF_WARPS) * 2 + 1) * d + c];
-      }
+      for (int j = 0; j < 4; ++j)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) { s0 += a[j]; s1 += b[j]; }
+        for (int q = 0; q < NS; ++q) a[j][q] = partial[((long)(k + j * CF_WARPS) * NS + q) * d + c];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int q = 0; q < NS; ++q) sv[q] += a[j][q];
     }
-    for (; k < nchunk; k += CF_WARPS) {
-      s0 += partial[((long)k * 2 + 0) * d + c];
-      s1 += partial[((long)k * 2 + 1) * d + c];
-    }
+    for (; k < nchunk; k += CF_WARPS)
+#pragma unroll
+      for (int q = 0; q < NS; ++q) sv[q] += partial[((long)k * NS + q) * d + c];
   }
-  red[0][warp][lane] = s0;
-  red[1][warp][lane] = s1;
+#pragma unroll
+  for (int q = 0; q < NS; ++q) red[q][warp][lane] = sv[q];
   __syncthreads();
   if (warp != 0 || c >= d) return;
-  s0 = s1 = 0.f;
 #pragma unroll
-  for (int w = 0; w < CF_WARPS; ++w) { s0 += red[0][w][lane]; s1 += red[1][w][lane]; }
-  if (accumulate) {
-    if (out0) out0[c] += s0;
-    if (out0b) out0b[c] += s0;
-    if (out1) out1[c] += s1;
-  } else {
-    if (out0) out0[c] = s0;
-    if (out0b) out0b[c] = s0;
-    if (out1) out1[c] = s1;
+  for (int q = 0; q < NS; ++q) {
+    sv[q] = 0.f;
+#pragma unroll
+    for (int w = 0; w < CF_WARPS; ++w) sv[q] += red[q][w][lane];
+  }
+  float* outs[5] = {out0, out0b, out1, NS > 2 ? out2 : nullptr, NS > 2 ? out2b : nullptr};
+  const int slot[5] = {0, 0, 1, NS > 2 ? 2 : 0, NS > 2 ? 2 : 0};
+#pragma unroll
+  for (int o = 0; o < 5; ++o) {
+    if (!outs[o]) continue;
+    outs[o][c] = accumulate ? outs[o][c] + sv[slot[o]] : sv[slot[o]];
   }
 }
 
@@ -554,26 +559,39 @@ int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
   int r = act_bf16 ? ln_bwd_t<bf16>(a, s) : ln_bwd_t<float>(a, s);
   count_launches(1);
   if (r) return r;
-  if (a.cs_part) {
+  if (a.cs_part && (a.cs_out1 || a.cs_out0)) {
     // column sums of the affine parameters' gradients by the separate reduction
     ColsumArgs c;
     memset(&c, 0, sizeof(c));
     c.rows = a.rows; c.d = a.d; c.src = a.dy; c.src_act = 0; c.ld = a.d; c.src2 = a.dy2;
     c.bmode = 1; c.x = a.x; c.mean = a.mean; c.rstd = a.rstd;
     c.partial = a.cs_part; c.out1 = a.cs_out1; c.out0 = a.cs_out0; c.accumulate = a.cs_accumulate;
-    return colsum(act_bf16, c, s);
+    if ((r = colsum(act_bf16, c, s)) != 0) return r;
+  }
+  if (a.cs_part && (a.dxs_out || a.dxs_out2)) {
+    // and of dx itself
+    ColsumArgs c;
+    memset(&c, 0, sizeof(c));
+    c.rows = a.rows; c.d = a.d; c.src = a.dx; c.src_act = 0; c.ld = a.d;
+    c.partial = a.cs_part; c.out0 = a.dxs_out; c.out0b = a.dxs_out2; c.accumulate = a.cs_accumulate;
+    if ((r = colsum(act_bf16, c, s)) != 0) return r;
   }
   return last_err();
 }
 
 int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* out0, float* out0b, int accumulate,
-                  cudaStream_t s) {
+                  cudaStream_t s, int nslot, float* out2, float* out2b) {
   if (d <= 0) return 0;
-  colsum_finish_kernel<<<(d + 31) / 32, CF_WARPS * 32, 0, s>>>(partial, nchunk, d, out1, out0, out0b, accumulate);
+  if (nslot == 3)
+    colsum_finish_kernel<3><<<(d + 31) / 32, CF_WARPS * 32, 0, s>>>(partial, nchunk, d, out1, out0, out0b, out2, out2b,
+                                                                     accumulate);
+  else
+    colsum_finish_kernel<2><<<(d + 31) / 32, CF_WARPS * 32, 0, s>>>(partial, nchunk, d, out1, out0, out0b, nullptr,
+                                                                     nullptr, accumulate);
   return last_err();
 }
 
-size_t colsum_partial_floats(int d) { return (size_t)kMaxColsumChunks * 2 * d; }
+size_t colsum_partial_floats(int d) { return (size_t)kMaxColsumChunks * 3 * d; }
 
 int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
   if (a.d <= 0) return 0;
@@ -605,8 +623,8 @@ int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s) {
   } else {
     colsum_kernel<float, 4><<<grid, CS_THREADS, 0, s>>>(a);
   }
-  colsum_finish_kernel<<<(a.d + 31) / 32, CF_WARPS * 32, 0, s>>>(a.partial, nch, a.d, a.out1, a.out0, a.out0b,
-                                                                  a.accumulate);
+  colsum_finish_kernel<2><<<(a.d + 31) / 32, CF_WARPS * 32, 0, s>>>(a.partial, nch, a.d, a.out1, a.out0, a.out0b,
+                                                                     nullptr, nullptr, a.accumulate);
   count_launches(2);
   return last_err();
 }

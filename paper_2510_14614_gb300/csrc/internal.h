@@ -92,11 +92,13 @@ struct LnFwdArgs {
   float* mean; float* rstd;             // [rows] or null
   // out2 = LN(x)*gamma+beta + add_src*add_g + add_b  (activation), if out2 != null
   void* out2; const float* add_src; const float* add_g; const float* add_b;
+  int* err;                             // receives DEV_ERR_TIMEOUT if a bounded wait expires (may be null)
 };
 int ln_fwd(int act_bf16, const LnFwdArgs& a, cudaStream_t s);
-// Sums nchunk per-chunk partial column sums [nchunk][2][d] into the outputs.
+// Sums nchunk per-chunk partial column sums [nchunk][nslot][d] into the
+// outputs (slot 0 -> out0 and out0b, slot 1 -> out1, slot 2 -> out2 and out2b).
 int colsum_finish(const float* partial, int nchunk, int d, float* out1, float* out0, float* out0b, int accumulate,
-                  cudaStream_t s);
+                  cudaStream_t s, int nslot = 2, float* out2 = nullptr, float* out2b = nullptr);
 
 struct LnBwdArgs {
   int rows, d;
@@ -109,7 +111,18 @@ struct LnBwdArgs {
   // rows: cs_out1 (+)= sum (dy + dy2) * xhat, cs_out0 (+)= sum (dy + dy2).
   // cs_part: scratch of colsum_partial_floats(d) floats.
   float* cs_part; float* cs_out1; float* cs_out0; int cs_accumulate;
+  // Optional column sums of the output dx itself (the bias gradients of the
+  // linear maps that produced the LN input's gradient): dxs_out and dxs_out2
+  // (+)= sum dx, with the same accumulate flag.  Needs cs_part.
+  float* dxs_out; float* dxs_out2;
+  int* err;                             // receives DEV_ERR_TIMEOUT if a bounded wait expires (may be null)
 };
+
+// Test hook for the bounded waits of the row-streaming LayerNorm kernels: when
+// stall_rows >= 0 each CTA's producer stops after that many rows, so that the
+// consumers' waits expire (after wait_ns, or the default budget when <= 0);
+// the kernels then report DEV_ERR_TIMEOUT and return.  stall_rows < 0: off.
+void ln_debug_stall(int stall_rows, long long wait_ns);
 int ln_bwd(int act_bf16, const LnBwdArgs& a, cudaStream_t s);
 // Row-streaming LayerNorm kernels (two persistent CTAs per SM, rows staged in
 // shared memory by bulk copies); 1 when the shape or alignment does not fit
@@ -130,7 +143,7 @@ struct ColsumArgs {
   int accumulate;                 // add into destinations instead of storing
 };
 int colsum(int act_bf16, const ColsumArgs& a, cudaStream_t s);
-size_t colsum_partial_floats(int d);  // = kMaxColsumChunks * 2 * d
+size_t colsum_partial_floats(int d);  // = kMaxColsumChunks * 3 * d
 constexpr int kMaxColsumChunks = 384;  // most per-chunk partials any column reduction writes
 
 int embed_fwd(int rows, int T, int d, int V, const int32_t* tok, const float* wte, const float* wpe,

@@ -16,9 +16,13 @@
 // pass over the rows is needed.
 //
 // Every mbarrier wait is bounded; on expiry the CTA's consumers agree (barrier
-// reduction) to stop, the producer waits for the copies it issued, and the
-// launch returns normally.  Two CTAs share an SM, so that one CTA's row
-// reductions overlap the other's.
+// reduction) to stop, record DEV_ERR_TIMEOUT in the device error word, the
+// producer waits for the copies it issued, and the launch returns normally.
+// Two CTAs share an SM, so that one CTA's row reductions overlap the other's.
+// The backward can also sum the columns of its output dx (the bias gradients
+// of the linear maps whose outputs feed the normalised residual).
+#include <atomic>
+
 #include "tc_ptx.cuh"
 
 namespace fal {
@@ -50,14 +54,31 @@ struct Ring {
   __device__ uint32_t empty(int s) const { return bar_base + 8u * (stages + s); }
 };
 
+// Bounded wait with a budget of wait_ns (the default when <= 0).
+__device__ __forceinline__ bool ring_wait(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag,
+                                          long long wait_ns) {
+  if (wait_ns <= 0) return mbar_wait(bar, parity, abort_flag);
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > (uint64_t)wait_ns) { *abort_flag = 1; return false; }
+  }
+}
+
 // One thread: copies every row r = blockIdx.x + k * gridDim.x of the sources
-// into the ring, then waits until each copy it issued has landed.
-__device__ void produce_rows(const RowSrc src, int rows, int d, const Ring ring, volatile uint32_t* abort_flag) {
+// into the ring, then waits until each copy it issued has landed (with the
+// default budget, whatever wait_ns is).  stall_rows >= 0 (test hook): stop
+// after that many rows.
+__device__ void produce_rows(const RowSrc src, int rows, int d, const Ring ring, volatile uint32_t* abort_flag,
+                             long long wait_ns, int stall_rows) {
   const uint32_t rb = (uint32_t)d * 4u;
-  int s = 0;
+  int s = 0, n = 0;
   uint32_t ph = 0, issued_mask = 0, issued_par = 0;
-  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
-    if (!mbar_wait(ring.empty(s), ph ^ 1u, abort_flag)) break;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x, ++n) {
+    if (stall_rows >= 0 && n >= stall_rows) break;
+    if (!ring_wait(ring.empty(s), ph ^ 1u, abort_flag, wait_ns)) break;
     mbar_arrive_expect_tx(ring.full(s), (uint32_t)src.n * rb);
     const uint32_t dst = ring.base + (uint32_t)s * ring.stage_bytes;
     for (int k = 0; k < src.n; ++k) bulk_load_1d(dst + (uint32_t)k * rb, src.p[k] + (long)r * d, rb, ring.full(s));
@@ -97,7 +118,8 @@ __device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 
 
 // y = LN(x) (* gamma + beta); optional fp32 copy; out2 = y + add_src * add_g + add_b.
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes) {
+__global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes,
+                                                                    long long wait_ns, int stall_rows) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
   volatile uint32_t* abort_flag;
@@ -110,7 +132,7 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdA
       RowSrc src;
       src.p[0] = a.x; src.p[1] = has2 ? a.add_src : nullptr; src.p[2] = src.p[3] = nullptr;
       src.n = has2 ? 2 : 1;
-      produce_rows(src, a.rows, d, ring, abort_flag);
+      produce_rows(src, a.rows, d, ring, abort_flag, wait_ns, stall_rows);
     }
     return;
   }
@@ -127,7 +149,7 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdA
   int s = 0;
   uint32_t ph = 0, it = 0;
   for (int r = blockIdx.x; r < a.rows; r += gridDim.x, ++it) {
-    const bool ok = mbar_wait(ring.full(s), ph, abort_flag);
+    const bool ok = ring_wait(ring.full(s), ph, abort_flag, wait_ns);
     float4 x[NCH], z[NCH];
     float sum = 0.f;
     const float4* st = reinterpret_cast<const float4*>(smem + (size_t)s * stage_bytes);
@@ -144,7 +166,10 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdA
     float* rb = red + (it & 1u) * 16;
     sum = warp_sum(sum);
     if (lane == 0) rb[warp] = sum;
-    if (named_bar_or(1, LR_CONS, !ok)) break;
+    if (named_bar_or(1, LR_CONS, !ok)) {
+      if (tid == 0) set_dev_err(a.err, DEV_ERR_TIMEOUT);
+      break;
+    }
     float tot = 0.f;
 #pragma unroll
     for (int w = 0; w < LR_WARPS; ++w) tot += rb[w];
@@ -187,7 +212,8 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdA
 // dx = rstd * (g - mean(g) - xhat * mean(g * xhat)) + dres with g = (dy + dy2) * gamma;
 // optional per-CTA column sums of (dy + dy2) * xhat and (dy + dy2).
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes) {
+__global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes,
+                                                                    long long wait_ns, int stall_rows) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
   volatile uint32_t* abort_flag;
@@ -203,22 +229,23 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdA
       src.n = 2;
       if (a.dy2) src.p[src.n++] = a.dy2;
       if (a.dres) src.p[src.n++] = a.dres;
-      produce_rows(src, a.rows, d, ring, abort_flag);
+      produce_rows(src, a.rows, d, ring, abort_flag, wait_ns, stall_rows);
     }
     return;
   }
-  float4 gam[NCH], cs0[NCH], cs1[NCH];
+  float4 gam[NCH], cs0[NCH], cs1[NCH], cs2[NCH];
+  const bool sum_dx = a.cs_part && (a.dxs_out || a.dxs_out2);
 #pragma unroll
   for (int k = 0; k < NCH; ++k) {
     const int c4 = tid + k * LR_CONS;
     gam[k] = (a.gamma && c4 < d4) ? load4(a.gamma + 4 * c4) : make_float4(1.f, 1.f, 1.f, 1.f);
-    cs0[k] = cs1[k] = f4_zero();
+    cs0[k] = cs1[k] = cs2[k] = f4_zero();
   }
   int s = 0;
   uint32_t ph = 0, it = 0;
   for (int r = blockIdx.x; r < a.rows; r += gridDim.x, ++it) {
     const float mean = a.mean[r], rstd = a.rstd[r];
-    const bool ok = mbar_wait(ring.full(s), ph, abort_flag);
+    const bool ok = ring_wait(ring.full(s), ph, abort_flag, wait_ns);
     float4 xh[NCH], gd[NCH], dr[NCH];
     float s1 = 0.f, s2 = 0.f;
     const float4* st = reinterpret_cast<const float4*>(smem + (size_t)s * stage_bytes);
@@ -247,7 +274,10 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdA
     s1 = warp_sum(s1);
     s2 = warp_sum(s2);
     if (lane == 0) { rb[warp] = s1; rb[8 + warp] = s2; }
-    if (named_bar_or(1, LR_CONS, !ok)) break;
+    if (named_bar_or(1, LR_CONS, !ok)) {
+      if (tid == 0) set_dev_err(a.err, DEV_ERR_TIMEOUT);
+      break;
+    }
     float m1 = 0.f, m2 = 0.f;
 #pragma unroll
     for (int w = 0; w < LR_WARPS; ++w) { m1 += rb[w]; m2 += rb[8 + w]; }
@@ -264,15 +294,18 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdA
                                    rstd * (gd[k].w - m1 - xh[k].w * m2) + dr[k].w);
       store4(a.dx + off + 4 * c4, o);
       if (a.dx_act) store4(reinterpret_cast<act_t*>(a.dx_act) + off + 4 * c4, o);
+      if (sum_dx) cs2[k] = f4_add(cs2[k], o);
     }
   }
   if (a.cs_part) {
+    const int ns = sum_dx ? 3 : 2;
 #pragma unroll
     for (int k = 0; k < NCH; ++k) {
       const int c4 = tid + k * LR_CONS;
       if (c4 >= d4) continue;
-      store4(a.cs_part + ((long)blockIdx.x * 2 + 0) * d + 4 * c4, cs0[k]);
-      store4(a.cs_part + ((long)blockIdx.x * 2 + 1) * d + 4 * c4, cs1[k]);
+      store4(a.cs_part + ((long)blockIdx.x * ns + 0) * d + 4 * c4, cs0[k]);
+      store4(a.cs_part + ((long)blockIdx.x * ns + 1) * d + 4 * c4, cs1[k]);
+      if (sum_dx) store4(a.cs_part + ((long)blockIdx.x * ns + 2) * d + 4 * c4, cs2[k]);
     }
   }
 }
@@ -292,6 +325,9 @@ bool set_smem_attr(K kernel) {
   return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LR_SMEM_MAX) == cudaSuccess;
 }
 
+std::atomic<int> g_stall_rows{-1};
+std::atomic<long long> g_wait_ns{0};
+
 int rows_grid(int rows) {
   int g = 2 * num_sms();
   if (g > kMaxColsumChunks) g = kMaxColsumChunks;  // per-CTA column partials must fit colsum_partial_floats(d)
@@ -308,8 +344,10 @@ int ln_fwd_rows(const LnFwdArgs& a, cudaStream_t s) {
   if (!st) return 1;
   const uint32_t smem = (uint32_t)st * sb + LR_TAIL_BYTES;
   const int grid = rows_grid(a.rows);
-  if (a.d <= 4 * LR_CONS) ln_fwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb);
-  else ln_fwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb);
+  const long long w = g_wait_ns.load();
+  const int sr = g_stall_rows.load();
+  if (a.d <= 4 * LR_CONS) ln_fwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else ln_fwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
   return 0;
 }
 
@@ -322,8 +360,10 @@ int ln_bwd_rows(const LnBwdArgs& a, cudaStream_t s) {
   if (!st) return 1;
   const uint32_t smem = (uint32_t)st * sb + LR_TAIL_BYTES;
   const int grid = rows_grid(a.rows);
-  if (a.d <= 4 * LR_CONS) ln_bwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb);
-  else ln_bwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb);
+  const long long w = g_wait_ns.load();
+  const int sr = g_stall_rows.load();
+  if (a.d <= 4 * LR_CONS) ln_bwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else ln_bwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
   return 0;
 }
 
@@ -342,8 +382,17 @@ int ln_bwd_bulk(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
     return 1;
   const int r = act_bf16 ? ln_bwd_rows<bf16>(a, s) : ln_bwd_rows<float>(a, s);
   if (r) return r;
-  if (a.cs_part) return colsum_finish(a.cs_part, rows_grid(a.rows), a.d, a.cs_out1, a.cs_out0, nullptr, a.cs_accumulate, s);
+  if (a.cs_part) {
+    const bool sum_dx = a.dxs_out || a.dxs_out2;
+    return colsum_finish(a.cs_part, rows_grid(a.rows), a.d, a.cs_out1, a.cs_out0, nullptr, a.cs_accumulate, s,
+                         sum_dx ? 3 : 2, a.dxs_out, a.dxs_out2);
+  }
   return 0;
+}
+
+void ln_debug_stall(int stall_rows, long long wait_ns) {
+  g_stall_rows.store(stall_rows);
+  g_wait_ns.store(wait_ns);
 }
 
 }  // namespace fal

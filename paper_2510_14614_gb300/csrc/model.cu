@@ -513,21 +513,29 @@ void ln_fwd_(Ctx& c, cudaStream_t s, const float* x, const float* gm, const floa
   memset(&a, 0, sizeof(a));
   a.rows = (int)c.h->BT; a.d = c.h->d; a.x = x; a.gamma = gm; a.beta = bt; a.out = out; a.out_f32 = out_f32;
   a.mean = mean; a.rstd = rstd; a.out2 = out2; a.add_src = add_src; a.add_g = add_g; a.add_b = add_b;
+  a.err = c.h->dev_err;
   ProfScope ps(c.h, s, 3, 0.0, "layernorm forward");
   c.check(ln_fwd(c.h->bf, a, s), "layernorm forward");
 }
 
+// Bias gradients that are column sums of a LayerNorm backward's output dx:
+// the linear maps whose outputs add into the residual that the LN normalised.
+struct BiasSum { float* b1 = nullptr; float* b2 = nullptr; };
+
 // LayerNorm backward; with dgamma/dbeta also the affine parameters' gradients
-// (column sums over the rows, computed in the same pass; part: scratch).
+// (column sums over the rows, computed in the same pass; part: scratch), and
+// with bias targets the column sums of dx itself, stored there.
 void ln_bwd_(Ctx& c, cudaStream_t s, const float* dy, const float* dy2, const float* x, const float* mean,
              const float* rstd, const float* gm, const float* dres, float* dx, void* dx_act, float* part = nullptr,
-             float* dgamma = nullptr, float* dbeta = nullptr) {
+             float* dgamma = nullptr, float* dbeta = nullptr, BiasSum bias = BiasSum()) {
   if (!c.ok()) return;
   LnBwdArgs a;
   memset(&a, 0, sizeof(a));
   a.rows = (int)c.h->BT; a.d = c.h->d; a.dy = dy; a.dy2 = dy2; a.x = x; a.mean = mean; a.rstd = rstd; a.gamma = gm;
   a.dres = dres; a.dx = dx; a.dx_act = dx_act;
-  if (dgamma || dbeta) { a.cs_part = part; a.cs_out1 = dgamma; a.cs_out0 = dbeta; }
+  a.err = c.h->dev_err;
+  if (dgamma || dbeta || bias.b1 || bias.b2) { a.cs_part = part; a.cs_out1 = dgamma; a.cs_out0 = dbeta; }
+  a.dxs_out = bias.b1; a.dxs_out2 = bias.b2;
   ProfScope ps(c.h, s, 3, 0.0, "layernorm backward");
   c.check(ln_bwd(c.h->bf, a, s), "layernorm backward");
 }
@@ -728,7 +736,7 @@ void mlp_backward(Ctx& c, int i, const float* dXn, const void* dXn_act, cudaStre
   gemm(c, group_calls({call1(d, F, wgrad_seg(h, dXn_act, d, A.g, F), wgrad_out(h, p.w_down, F)),
                        call1(BT, F, dgrad_seg(h, dXn_act, d, p.w_down, F), e)}),
        s, "MLP down wgrad + dgrad");
-  colsum_(c, s, part, dXn, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_down), nullptr, 0);
+  (void)dXn;  // db_down = column sums of dXn, summed by the LayerNorm backward that produced it
   gemm(c, group_calls({call1(F, d, wgrad_seg(h, h->dh, F, mlp_in(h, i), d), wgrad_out(h, p.w_up, d)),
                        call1(BT, d, dgrad_seg(h, h->dh, F, p.w_up, d), epi_out(h->dU2, d, OUT_F32))}),
        s, "MLP up wgrad + dgrad");
@@ -752,7 +760,7 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
     gemm(c, group_calls({call1(d, d, wgrad_seg(h, da_act, d, A.ctx, d), wgrad_out(h, p.w_o, d)),
                          call1(BT, d, dgrad_seg(h, da_act, d, p.w_o, d), edc)}),
          s, "attention out wgrad + dgrad");
-    colsum_(c, s, part, da, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o), nullptr, 0);
+    (void)da;  // db_o = column sums of da, summed by the LayerNorm backward that produced it
   }
   if (!c.ok()) return;
   h->err.clear();
@@ -783,6 +791,19 @@ void first_attention_grad(Ctx& c, size_t g_off, size_t b_off, cudaStream_t s, fl
           Gp(h, g_off), Gp(h, b_off), nullptr, accumulate);
 }
 
+// The bias gradients of block j that are column sums of dX_{j+1} (the gradient
+// of the block's output): b_down, and for blocks whose branches both add into
+// the residual at once (Parallel-type), b_o too.  Summed by the LayerNorm
+// backward that produces dX_{j+1}.
+BiasSum down_biases(fal_handle* h, int j) {
+  BiasSum b;
+  if (j < 0) return b;
+  const LayerP& p = h->lp[j];
+  b.b1 = Gp(h, p.b_down);
+  if (block_kind(h, j) == BK_PAR) b.b2 = Gp(h, p.b_o);
+  return b;
+}
+
 void layer_backward(Ctx& c, int i) {
   fal_handle* h = c.h;
   LayerA& A = h->la[i];
@@ -806,8 +827,7 @@ void layer_backward(Ctx& c, int i) {
                          call1(BT, d, dgrad_seg(h, h->dX_act, d, p.w_o, d), edc),
                          call1(BT, F, dgrad_seg(h, h->dX_act, d, p.w_down, F), edh)}),
          s, "fused residual wgrad + dgrad");
-    colsum_(c, s, h->part0, h->dX, 0, d, d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_o),
-            Gp(h, p.b_down), 0);
+    // (db_o = db_down = column sums of dX, summed by the LayerNorm backward that produced dX)
     const bool two = h->cfg.schedule == FAL_SCHED_TWO_STREAM && h->ss != h->sm;
     cudaStream_t sa = two ? h->ss : s;
     if (two) fork(h);
@@ -820,7 +840,7 @@ void layer_backward(Ctx& c, int i) {
     if (var == FAL_FAL) first_attention_grad(c, h->lnF_g, h->lnF_b, s, h->part0, 1);
     if (two) join(h);
     ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
-            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
+            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b), down_biases(h, i - 1));
     return;
   }
   if (kind == BK_FIRST || kind == BK_OWN) {  // FAL block 1, Ablation1 blocks
@@ -834,27 +854,31 @@ void layer_backward(Ctx& c, int i) {
     }
     // da = dX_{i+1} + (LN without affine)'(a) . dA1hat   (a feeds X_{i+1} and the MLP input)
     ln_bwd_(c, s, h->dA1hat, nullptr, first ? h->a1 : A.a, first ? h->a1_mean : A.a_mean,
-            first ? h->a1_rstd : A.a_rstd, nullptr, h->dX, h->dA, h->dA_act);
+            first ? h->a1_rstd : A.a_rstd, nullptr, h->dX, h->dA, h->dA_act, h->part0, nullptr, nullptr,
+            BiasSum{Gp(h, p.b_o), nullptr});
     attn_backward(c, i, h->dA, h->dA_act, s, h->part0, false);
     ln_bwd_(c, s, h->dU, h->dU2, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dX, h->dX, h->dX_act,
-            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
+            h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b), down_biases(h, i - 1));
     return;
   }
   // GPT / FAL+
   mlp_backward(c, i, h->dX, h->dX_act, s, h->part0);
+  // db_o = column sums of da: dY here, or dA for the block whose attention FAL+ reuses
+  const bool reused = var == FAL_FALPLUS && i == h->reuse;
   ln_bwd_(c, s, h->dU2, nullptr, A.Y, A.ln2_mean, A.ln2_rstd, Pp(h, p.ln2_g), h->dX, h->dY, h->dY_act,
-          h->part0, Gp(h, p.ln2_g), Gp(h, p.ln2_b));
+          h->part0, Gp(h, p.ln2_g), Gp(h, p.ln2_b), reused ? BiasSum() : BiasSum{Gp(h, p.b_o), nullptr});
   const float* da = h->dY;
   const void* da_act = h->dY_act;
   if (var == FAL_FALPLUS && i > h->reuse) first_attention_grad(c, p.lnF_g, p.lnF_b, s, h->part0, 0);
   if (var == FAL_FALPLUS && i == h->reuse) {
-    ln_bwd_(c, s, h->dA1hat, nullptr, h->a1, h->a1_mean, h->a1_rstd, nullptr, h->dY, h->dA, h->dA_act);
+    ln_bwd_(c, s, h->dA1hat, nullptr, h->a1, h->a1_mean, h->a1_rstd, nullptr, h->dY, h->dA, h->dA_act, h->part0,
+            nullptr, nullptr, BiasSum{Gp(h, p.b_o), nullptr});
     da = h->dA;
     da_act = h->dA_act;
   }
   attn_backward(c, i, da, da_act, s, h->part0, false);
   ln_bwd_(c, s, h->dU, nullptr, A.X, A.ln1_mean, A.ln1_rstd, Pp(h, p.ln1_g), h->dY, h->dX, h->dX_act,
-          h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b));
+          h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b), down_biases(h, i - 1));
 }
 
 int backward_impl(fal_handle* h) {
@@ -867,7 +891,7 @@ int backward_impl(fal_handle* h) {
                        call1(BT, d, seg(h->dlogits, h->Vp, 0, Wp(h, h->wte), d, 1, h->V), epi_out(h->dU, d, OUT_F32))}),
        s, "LM head wgrad + dgrad");
   ln_bwd_(c, s, h->dU, nullptr, h->Xout, h->lnf_mean, h->lnf_rstd, Pp(h, h->lnf_g), nullptr, h->dX, h->dX_act,
-          h->part0, Gp(h, h->lnf_g), Gp(h, h->lnf_b));
+          h->part0, Gp(h, h->lnf_g), Gp(h, h->lnf_b), down_biases(h, h->L - 1));
   if (h->cfg.variant != FAL_GPT) cudaMemsetAsync(h->dA1hat, 0, (size_t)BT * d * 4, s);
   if (h->cfg.variant == FAL_FAL) {
     cudaMemsetAsync(Gp(h, h->lnF_g), 0, (size_t)d * 4, s);
@@ -1242,6 +1266,11 @@ int fal_profile_read(fal_handle* h, fal_profile* out) {
 }
 
 long long fal_launch_count(void) { return launches_total(); }
+
+int fal_debug_layernorm_stall(int rows, long long wait_ns) {
+  ln_debug_stall(rows < 0 ? -1 : rows, wait_ns > 0 ? wait_ns : 0);
+  return FAL_OK;
+}
 
 const char* fal_last_error(const fal_handle* h) {
   if (!h) return "null handle";

@@ -79,6 +79,7 @@ _SIGS = {
     "fal_profile_timeline": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(FalLaunchRecord), ctypes.c_int,
                                             ctypes.POINTER(ctypes.c_int)]),
     "fal_launch_count": (ctypes.c_longlong, []),
+    "fal_debug_layernorm_stall": (ctypes.c_int, [ctypes.c_int, ctypes.c_longlong]),
     "fal_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),
     "fal_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "fal_kernel_gemm": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_long,

@@ -307,3 +307,32 @@ def test_split_k_residual_is_reproducible():
     m.forward(tok, tgt)
     for i, x in enumerate(first, start=1):
         np.testing.assert_array_equal(m.tap("X", i), x, err_msg=f"X{i}")
+
+
+@pytest.mark.parametrize("stall_rows", [0, 1])
+def test_bounded_wait_expiry_is_reported_and_the_handle_recovers(stall_rows):
+    """The row-streaming LayerNorm kernels' producers stop after `stall_rows`
+    rows per CTA (test hook; B*T = 1200 rows give every CTA about four), so
+    their consumers wait for rows that never come: the bounded waits expire
+    after 2 ms, the kernels record a timeout and return, and the forward
+    reports FAL_ERR_TIMEOUT.  With the hook off again the same handle gives the
+    bitwise same loss as before and still trains."""
+    from paper_2510_14614_gb300 import fal
+    s = SMALL.replace(layers=2, seq=600)
+    params = synth.perturb_params(synth.init_params("fal", s, 6), 6)
+    tok, tgt = synth.make_tokens(s, 6)
+    m = _model("fal", s, "two_stream")
+    m.set_params(params)
+    before = m.forward(tok, tgt)
+    lib = fal.lib()
+    try:
+        assert lib.fal_debug_layernorm_stall(stall_rows, 2_000_000) == fal.FAL_OK
+        with pytest.raises(fal.FalError) as e:
+            m.forward(tok, tgt)
+        assert e.value.code == fal.FAL_ERR_TIMEOUT
+    finally:
+        lib.fal_debug_layernorm_stall(-1, 0)
+    assert m.forward(tok, tgt) == before
+    m.backward()
+    m.step()
+    assert np.isfinite(m.train_step(tok, tgt))
