@@ -22,6 +22,9 @@ One JSON line carries, besides the headline (timed with profiling off):
                 FAL+ beside GPT, tokens/s and fraction of peak;
   attention_isolated  forward and backward attention kernels timed alone on one
                 layer of the headline shape;
+  inference     forward-only prefill (App. E: forward step without gradients,
+                the time to first token) of FAL and GPT at the headline shape
+                and for single requests of 2048 and 1024 tokens;
   cpu_baseline  a measured sample of one fp64 oracle training step (OracleSample).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
@@ -66,6 +69,7 @@ def parse(argv=None):
     ap.add_argument("--no-baseline", action="store_true", help="skip the GPT and FAL-serial arms of the headline shape")
     ap.add_argument("--no-configs", action="store_true", help="skip the other benchmark shapes")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--no-inference", action="store_true", help="skip the forward-only prefill arms")
     ap.add_argument("--arm-steps", type=int, default=5, help="timed steps of each extra arm")
     ap.add_argument("--layers", type=int, default=None, help="override depth (small profiling cases only)")
     ap.add_argument("--batch", type=int, default=None, help="override batch (small profiling cases only)")
@@ -353,6 +357,21 @@ class Arm:
             out["clocks"] = clk.summary()
         return out
 
+    def prefill_ms(self, steps, warmup):
+        """Forward-only prefill (no loss, no backward state), CUDA events on the
+        library's main stream."""
+        torch = self.torch
+        for _ in range(warmup):
+            self.m.prefill(self.tok, sync=False)
+        torch.cuda.synchronize(self.dev)
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(self.m.stream_main)
+        for _ in range(steps):
+            self.m.prefill(self.tok, sync=False)
+        ev1.record(self.m.stream_main)
+        torch.cuda.synchronize(self.dev)
+        return ev0.elapsed_time(ev1) / steps
+
     def e2e(self, steps, world):
         """Through the public C ABI with host buffers: pinned token upload, the
         step, and the loss read back to the host every step."""
@@ -553,6 +572,25 @@ def main():
             cfgs[name] = row
         out["configs"] = cfgs
         out["configs_note"] = f"{w} warm-up and {k} timed steps per arm; fractions against measured burst / sustained"
+    if not args.no_inference and extra and args.layers is None and args.batch is None:
+        inf = {}
+        for label, shp in (("batch", s), ("request_T2048", s.replace(batch=1, seq=min(2048, s.seq))),
+                           ("request_T1024", s.replace(batch=1, seq=min(1024, s.seq)))):
+            row = {}
+            for v, sched in ((args.variant, args.schedule), ("gpt", "serial")):
+                if v in row:
+                    continue
+                a = Arm(shp, v, sched, torch, fal, dev, rank)
+                ms_pf = a.prefill_ms(10, 3)
+                a.close()
+                row[variant_name(v)] = {"ms": ms_pf, "tokens_per_s": shp.tokens / (ms_pf / 1e3), "schedule": sched}
+            if "GPT" in row and variant_name(args.variant) in row and args.variant != "gpt":
+                row[f"{variant_name(args.variant)}/GPT"] = row["GPT"]["ms"] / row[variant_name(args.variant)]["ms"]
+            row["shape"] = f"batch={shp.batch} seq={shp.seq}"
+            inf[label] = row
+        out["inference"] = inf
+        out["inference_note"] = ("fal_prefill: embedding, every block, final LN and the LM head of each sequence's "
+                                 "last position; 3 warm-up and 10 timed calls, CUDA events")
     if rank == 0 and n == 1 and not args.no_cpu:
         cpu = OracleSample(s, args.variant, 1, min(CPU_SEQ, s.seq))
         sec = cpu()

@@ -119,6 +119,15 @@ void fal_destroy(fal_handle* h);
  * reported as FAL_ERR_ARG at the next synchronizing call. */
 int fal_forward(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host);
 
+/* Forward-only pass for inference, the paper's "forward step time without
+ * gradient calculation" that matches the time to first token (App. E): the
+ * stack over tokens [B, T] (int32 row-major, device or host), the final
+ * LayerNorm, and the tied LM head for the last position of every sequence
+ * only.  last_logits: fp32 [B, V] row-major, device or host, or NULL to leave
+ * them on the device; a non-NULL pointer makes the call synchronize.  No loss
+ * and no backward state: a following fal_backward returns FAL_ERR_STATE. */
+int fal_prefill(fal_handle* h, const int32_t* tokens, float* last_logits);
+
 /* Gradients of the last forward's loss into the flat fp32 gradient buffer
  * (overwritten, not accumulated).  FAL_ERR_STATE without a preceding forward. */
 int fal_backward(fal_handle* h);

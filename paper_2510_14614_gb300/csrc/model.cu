@@ -1031,6 +1031,38 @@ int fal_forward(fal_handle* h, const int32_t* tokens, const int32_t* targets, fl
   return FAL_OK;
 }
 
+int fal_prefill(fal_handle* h, const int32_t* tokens, float* last_logits) {
+  if (!h || !tokens) return h ? fail(h, FAL_ERR_ARG, "null tokens") : FAL_ERR_ARG;
+  Ctx c{h};
+  cudaStream_t s = h->sm;
+  const int d = h->d;
+  if (cudaMemcpyAsync(h->tok, tokens, (size_t)h->BT * sizeof(int32_t), cudaMemcpyDefault, s) != cudaSuccess)
+    return fail(h, FAL_ERR_CUDA, "token copy failed");
+  h->state = 0;  // the saved activations are overwritten: no backward after this
+  c.check(embed_fwd((int)h->BT, h->T, d, h->V, h->tok, Pp(h, h->wte), Pp(h, h->wpe), h->la[0].X, h->dev_err, s),
+          "embedding");
+  for (int i = 0; i < h->L && c.ok(); ++i) layer_forward(c, i);
+  ln_fwd_(c, s, h->Xout, Pp(h, h->lnf_g), Pp(h, h->lnf_b), h->xf, nullptr, h->lnf_mean, h->lnf_rstd, nullptr, nullptr,
+          nullptr, nullptr);
+  // LM head on the last position of every sequence: rows T-1, 2T-1, ... of xf
+  // (row pitch T*d), fp32 logits [B, Vp] in the staging buffer when they fit,
+  // else in the logits buffer (B*Vp fp32 values fit there when T >= 2)
+  const size_t need = (size_t)h->B * h->Vp;
+  float* out = need <= h->stage_floats ? h->stage : reinterpret_cast<float*>(h->logits);
+  if (out != h->stage && h->bf && h->T < 2) return fail(h, FAL_ERR_UNSUPPORTED, "prefill logits do not fit the workspace");
+  const uint8_t* last = reinterpret_cast<const uint8_t*>(h->xf) + (size_t)(h->T - 1) * d * h->asz;
+  gemm(c, call1(h->B, h->V, seg(last, (long)h->T * d, 0, Wp(h, h->wte), d, 0, d), epi_out(out, h->Vp, OUT_F32)), s,
+       "LM head (last positions)");
+  if (!c.ok()) return c.rc;
+  if (last_logits) {
+    if (cudaMemcpy2DAsync(last_logits, (size_t)h->V * 4, out, (size_t)h->Vp * 4, (size_t)h->V * 4, h->B,
+                          cudaMemcpyDefault, s) != cudaSuccess)
+      return fail(h, FAL_ERR_CUDA, "logits copy failed");
+    return read_dev_err(h);
+  }
+  return FAL_OK;
+}
+
 int fal_backward(fal_handle* h) {
   if (!h) return FAL_ERR_ARG;
   if (h->state < 1) return fail(h, FAL_ERR_STATE, "fal_backward needs a preceding fal_forward");

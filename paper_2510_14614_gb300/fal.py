@@ -59,6 +59,7 @@ _SIGS = {
     "fal_destroy": (None, [ctypes.c_void_p]),
     "fal_forward": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "fal_backward": (ctypes.c_int, [ctypes.c_void_p]),
+    "fal_prefill": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "fal_step": (ctypes.c_int, [ctypes.c_void_p]),
     "fal_train_step": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(ctypes.c_float)]),
     "fal_sync": (ctypes.c_int, [ctypes.c_void_p]),
@@ -242,6 +243,17 @@ class Model:
         loss = ctypes.c_float()
         _check(lib().fal_forward(self.h, t, g, ctypes.byref(loss) if sync else None), self.h, "fal_forward")
         return loss.value if sync else None
+
+    def prefill(self, tokens, sync=True):
+        """Forward-only pass; returns the fp32 logits [B, V] of every sequence's
+        last position (sync=True), or None with the work left queued."""
+        t, _ = self._tokens(tokens, tokens)
+        if not sync:
+            _check(lib().fal_prefill(self.h, t, None), self.h, "fal_prefill")
+            return None
+        out = np.empty((self.cfg.batch, self.cfg.vocab), np.float32)
+        _check(lib().fal_prefill(self.h, t, out.ctypes.data_as(ctypes.c_void_p)), self.h, "fal_prefill")
+        return out
 
     def backward(self):
         _check(lib().fal_backward(self.h), self.h, "fal_backward")

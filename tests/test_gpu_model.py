@@ -336,3 +336,28 @@ def test_bounded_wait_expiry_is_reported_and_the_handle_recovers(stall_rows):
     m.backward()
     m.step()
     assert np.isfinite(m.train_step(tok, tgt))
+
+
+@pytest.mark.parametrize("variant,shape,schedule", [("fal", "small", "two_stream"), ("gpt", "small", "serial"),
+                                                    ("falplus", "hd128", "serial"), ("fal", "tiny", "serial"),
+                                                    ("parallel", "small", "two_stream")])
+def test_prefill_last_logits_match_oracle(variant, shape, schedule):
+    """Forward-only prefill (App. E inference): the logits of every sequence's
+    last position against the oracle's forward; no backward state after it."""
+    from paper_2510_14614_gb300 import fal
+    s = {"small": SMALL, "hd128": HD128}.get(shape) or synth.SHAPES["tiny"].replace(layers=3)
+    params = synth.perturb_params(synth.init_params(variant, s, 8), 8)
+    tok, tgt = synth.make_tokens(s, 8)
+    m = _model(variant, s, schedule)
+    m.set_params(params)
+    got = m.prefill(tok)
+    _, cache = O.forward(params, O.Config.from_shape(variant, s), tok, tgt)
+    ref = cache["logits"].reshape(s.batch, s.seq, s.vocab)[:, -1, :]
+    tol = 1e-2 if s.precision == "bf16" else 1e-4
+    assert got.shape == (s.batch, s.vocab)
+    assert rel_fro(got, ref) <= tol, rel_fro(got, ref)
+    with pytest.raises(fal.FalError) as e:
+        m.backward()
+    assert e.value.code == fal.FAL_ERR_STATE
+    # a training step after the prefill still works
+    assert np.isfinite(m.train_step(tok, tgt))
