@@ -17,6 +17,10 @@ NumPy (matmul is the only library primitive used):
   * FAL+ block (Sec. 5; App. D.1 equation): block 1 is the standard block;
     block i >= 2 feeds MLP_i(LN(X_i + MHA_i(LN(X_i))) + LN_{F,i}(MHA_1(LN(X_1))))
     with its own LayerNorm LN_{F,i} on the first attention output.
+  * Grouped-query attention (App. E, GQA): with G key/value heads, query head
+    h attends with the key and value head of its group h // (H / G); G = H is
+    multi-head attention.  The fused QKV projection then has d_model query
+    columns and G * head_dim key and value columns each.
   * GPT-2 conventions (the paper builds on GPT-2, Sec. 5.1): learned position
     embedding, tied LM head, final LayerNorm, biases on every linear map,
     tanh-approximated GELU, LayerNorm eps 1e-5 with the population variance,
@@ -125,7 +129,8 @@ VARIANTS = ("gpt", "fal", "falplus", "parallel", "ablation1", "ablation2")
 
 
 class Config:
-    def __init__(self, variant, layers, d_model, heads, d_ff, seq, batch, vocab, reuse=1, separate_ln2=False):
+    def __init__(self, variant, layers, d_model, heads, d_ff, seq, batch, vocab, reuse=1, separate_ln2=False,
+                 kv_heads=0):
         assert variant in VARIANTS
         assert d_model % heads == 0
         assert reuse >= 1 and (reuse == 1 or variant == "falplus")
@@ -133,10 +138,13 @@ class Config:
         self.variant, self.layers, self.d_model, self.heads = variant, layers, d_model, heads
         self.d_ff, self.seq, self.batch, self.vocab = d_ff, seq, batch, vocab
         self.reuse, self.separate_ln2 = reuse, separate_ln2
+        self.kv_heads = kv_heads or heads
+        assert heads % self.kv_heads == 0
 
     @classmethod
     def from_shape(cls, variant, s, **kw):
-        return cls(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab, **kw)
+        return cls(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
+                   kv_heads=getattr(s, "kv_heads", 0), **kw)
 
 
 def _split_heads(x, B, T, H):
@@ -166,8 +174,12 @@ def forward(params, cfg, tokens, targets, layers=None):
         c = {}
         u, c["ln1"] = layer_norm(X, w("ln1.g"), w("ln1.b"))
         qkv = u @ w("attn.w_qkv").T + w("attn.b_qkv")
-        q, k, v = (_split_heads(t, B, T, H) for t in np.split(qkv, 3, axis=1))
-        o, p = causal_attention(q, k, v)
+        nkv = cfg.kv_heads
+        q = _split_heads(qkv[:, :d], B, T, H)
+        k = _split_heads(qkv[:, d:d + nkv * (d // H)], B, T, nkv)
+        v = _split_heads(qkv[:, d + nkv * (d // H):], B, T, nkv)
+        # every query head uses the key / value head of its group
+        o, p = causal_attention(q, np.repeat(k, H // nkv, axis=1), np.repeat(v, H // nkv, axis=1))
         ctx = _merge_heads(o)
         a = ctx @ w("attn.w_o").T + w("attn.b_o")
         if i == k_reuse:
@@ -263,7 +275,12 @@ def backward(params, cfg, cache):
         G[gn("attn.w_o")] = da.T @ c["ctx"]
         G[gn("attn.b_o")] = da.sum(0)
         dctx = _split_heads(da @ w("attn.w_o"), B, T, H)
-        dq, dk, dv = causal_attention_backward(dctx, c["q"], c["k"], c["v"], c["p"])
+        nkv = cfg.kv_heads
+        dq, dk, dv = causal_attention_backward(dctx, c["q"], np.repeat(c["k"], H // nkv, axis=1),
+                                               np.repeat(c["v"], H // nkv, axis=1), c["p"])
+        # a key / value head's gradient sums over the query heads of its group
+        dk = dk.reshape(B, nkv, H // nkv, T, -1).sum(2)
+        dv = dv.reshape(B, nkv, H // nkv, T, -1).sum(2)
         dqkv = np.concatenate([_merge_heads(dq), _merge_heads(dk), _merge_heads(dv)], axis=1)
         G[gn("attn.w_qkv")] = dqkv.T @ c["u"]
         G[gn("attn.b_qkv")] = dqkv.sum(0)

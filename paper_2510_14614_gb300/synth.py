@@ -41,10 +41,21 @@ class Shape:
     vocab: int
     precision: str  # "fp32" (debug path) or "bf16"
     scale_out_proj: bool = False
+    kv_heads: int = 0  # key/value heads (GQA groups); 0 = one per query head (MHA)
 
     @property
     def head_dim(self) -> int:
         return self.d_model // self.heads
+
+    @property
+    def kv(self) -> int:
+        return self.kv_heads or self.heads
+
+    @property
+    def d_qkv(self) -> int:
+        """Width of the fused QKV projection: d_model query columns and kv * head_dim
+        key and value columns each."""
+        return self.d_model + 2 * self.kv * self.head_dim
 
     @property
     def tokens(self) -> int:
@@ -88,12 +99,13 @@ def param_specs(variant: str, s: Shape, reuse: int = 1, separate_ln2: bool = Fal
     if reuse < 1 or (reuse != 1 and variant != "falplus") or (separate_ln2 and variant != "fal"):
         raise ValueError("reuse applies to FAL+ and separate_ln2 to FAL")
     d, f, V, T, L = s.d_model, s.d_ff, s.vocab, s.seq, s.layers
+    dq = s.d_qkv
     specs = [("wte", (V, d), True), ("wpe", (T, d), True)]
     for i in range(L):
         p = f"h{i}."
         specs += [
             (p + "ln1.g", (d,), False), (p + "ln1.b", (d,), False),
-            (p + "attn.w_qkv", (3 * d, d), True), (p + "attn.b_qkv", (3 * d,), False),
+            (p + "attn.w_qkv", (dq, d), True), (p + "attn.b_qkv", (dq,), False),
             (p + "attn.w_o", (d, d), True), (p + "attn.b_o", (d,), False),
         ]
         if variant in ("gpt", "falplus") or (variant == "ablation2" and i == 0) or separate_ln2:

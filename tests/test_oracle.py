@@ -472,3 +472,70 @@ def test_clip_grad_norm_matches_torch(max_norm):
     else:
         total = math.sqrt(sum(float((c ** 2).sum()) for c in clipped.values()))
         assert abs(total - max_norm) < 1e-12 * max_norm
+
+
+# ------------------------------------------------------------------ grouped-query attention
+GQA = [("fal", 2), ("gpt", 2), ("falplus", 1), ("fal", 4)]  # (variant, key/value heads) with H = 4
+
+
+@pytest.mark.parametrize("variant,kv", GQA)
+def test_gqa_matches_autograd_model(variant, kv):
+    """App. E: GQA with G key/value heads; the torch model repeats each
+    key / value head over its H / G query heads and differentiates by autograd."""
+    s = TINY.replace(layers=3, kv_heads=kv)
+    p = synth.perturb_params(synth.init_params(variant, s, 31), 31)
+    assert p["h0.attn.w_qkv"].shape == (s.d_model + 2 * kv * s.head_dim, s.d_model)
+    tok, tgt = synth.make_tokens(s, 12)
+    cfg = O.Config.from_shape(variant, s)
+    loss, cache = O.forward(p, cfg, tok, tgt)
+    grads = O.backward(p, cfg, cache)
+    tloss, tgrads = torch_ref.loss_and_grads(p, variant, s.heads, tok, tgt, s.layers, kv_heads=kv)
+    assert abs(loss - tloss) < 1e-12
+    for k in p:
+        np.testing.assert_allclose(grads[k], tgrads[k], rtol=1e-9, atol=1e-13, err_msg=k)
+
+
+@pytest.mark.parametrize("variant,kv", GQA[:2])
+def test_gqa_backward_matches_central_differences(variant, kv):
+    s = TINY.replace(layers=2, kv_heads=kv)
+    p = {k: a.astype(np.float64) for k, a in synth.perturb_params(synth.init_params(variant, s, 32), 32).items()}
+    tok, tgt = synth.make_tokens(s, 13)
+    cfg = O.Config.from_shape(variant, s)
+    _, cache = O.forward(p, cfg, tok, tgt)
+    grads = O.backward(p, cfg, cache)
+    rng = np.random.default_rng(33)
+    h = 1e-5
+    for k in p:
+        direction = rng.standard_normal(p[k].shape)
+        direction /= np.linalg.norm(direction)
+        pp, pm = dict(p), dict(p)
+        pp[k], pm[k] = p[k] + h * direction, p[k] - h * direction
+        fd = (O.loss_only(pp, cfg, tok, tgt) - O.loss_only(pm, cfg, tok, tgt)) / (2 * h)
+        an = float((grads[k] * direction).sum())
+        assert abs(fd - an) <= 1e-6 * np.linalg.norm(grads[k]) + 1e-11, (k, fd, an)
+
+
+def test_gqa_with_one_group_per_head_is_mha_and_shared_kv_acts_as_copies():
+    """G = H is multi-head attention (App. E); and a GQA model equals the MHA
+    model whose key / value projections repeat the group's rows for each of
+    its query heads."""
+    s = TINY.replace(layers=2)
+    p = _params("fal", s, seed=34)
+    tok, tgt = synth.make_tokens(s, 14)
+    l_mha, _ = O.forward(p, O.Config.from_shape("fal", s), tok, tgt)
+    l_g, _ = O.forward(p, O.Config.from_shape("fal", s.replace(kv_heads=s.heads)), tok, tgt)
+    assert l_mha == l_g
+    sg = s.replace(kv_heads=2)
+    pg = synth.perturb_params(synth.init_params("fal", sg, 35), 35)
+    d, hd, H = s.d_model, s.head_dim, s.heads
+    pm = dict(pg)
+    for i in range(s.layers):
+        w, b = pg[f"h{i}.attn.w_qkv"], pg[f"h{i}.attn.b_qkv"]
+        kw, vw = w[d:d + 2 * hd], w[d + 2 * hd:]
+        kb, vb = b[d:d + 2 * hd], b[d + 2 * hd:]
+        rep = lambda a: np.concatenate([a[(h // (H // 2)) * hd:(h // (H // 2) + 1) * hd] for h in range(H)], axis=0)
+        pm[f"h{i}.attn.w_qkv"] = np.concatenate([w[:d], rep(kw), rep(vw)], axis=0)
+        pm[f"h{i}.attn.b_qkv"] = np.concatenate([b[:d], rep(kb), rep(vb)], axis=0)
+    l1, _ = O.forward(pg, O.Config.from_shape("fal", sg), tok, tgt)
+    l2, _ = O.forward(pm, O.Config.from_shape("fal", s), tok, tgt)
+    assert abs(l1 - l2) < 1e-12

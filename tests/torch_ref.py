@@ -17,12 +17,16 @@ def _ln(x, p, name):
     return Fn.layer_norm(x, (d,), p[name + ".g"], p[name + ".b"], eps=1e-5)
 
 
-def _mha(x, p, i, H):
+def _mha(x, p, i, H, G=None):
     B, T, d = x.shape
+    G = G or H
+    hd = d // H
     qkv = Fn.linear(x, p[f"h{i}.attn.w_qkv"], p[f"h{i}.attn.b_qkv"])
-    q, k, v = qkv.split(d, dim=-1)
-    sh = lambda t: t.reshape(B, T, H, d // H).transpose(1, 2)
-    o = Fn.scaled_dot_product_attention(sh(q), sh(k), sh(v), is_causal=True)
+    q, k, v = qkv.split([d, G * hd, G * hd], dim=-1)
+    sh = lambda t, n: t.reshape(B, T, n, hd).transpose(1, 2)
+    # grouped-query attention: each key / value head serves H / G query heads
+    rep = lambda t: sh(t, G).repeat_interleave(H // G, dim=1)
+    o = Fn.scaled_dot_product_attention(sh(q, H), rep(k), rep(v), is_causal=True)
     o = o.transpose(1, 2).reshape(B, T, d)
     return Fn.linear(o, p[f"h{i}.attn.w_o"], p[f"h{i}.attn.b_o"])
 
@@ -32,7 +36,8 @@ def _mlp(x, p, i):
     return Fn.linear(Fn.gelu(h, approximate="tanh"), p[f"h{i}.mlp.w_down"], p[f"h{i}.mlp.b_down"])
 
 
-def model_loss(params, variant, heads, tokens, targets, layers, parallel=False, reuse=1, separate_ln2=False):
+def model_loss(params, variant, heads, tokens, targets, layers, parallel=False, reuse=1, separate_ln2=False,
+               kv_heads=None):
     """Mean next-token loss.  ``parallel=True`` builds the GPT-J style block
     X + MHA(LN1(X)) + MLP(LN1(X)) (no first-attention term), as does the
     variant "parallel"; "ablation1" / "ablation2" are App. D's ablations;
@@ -45,7 +50,7 @@ def model_loss(params, variant, heads, tokens, targets, layers, parallel=False, 
     a1 = None
     for i in range(layers):
         n1 = _ln(X, p, f"h{i}.ln1")
-        a = _mha(n1, p, i, heads)
+        a = _mha(n1, p, i, heads, kv_heads)
         if i == reuse - 1:
             a1 = a
         if parallel or variant == "parallel" or (variant == "ablation2" and i >= 1):
