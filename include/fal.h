@@ -83,6 +83,9 @@ typedef struct fal_config {
                          clipping, fal_train_step cannot update weights inside the gradient
                          GEMMs (the norm needs every gradient first) and runs AdamW after
                          the backward, like fal_step. */
+    int kv_heads;     /* grouped-query attention (App. E): key/value heads, each shared by
+                         heads / kv_heads query heads; 0 = heads (multi-head attention).
+                         The fused QKV matrix then has d_model + 2 * kv_heads * head_dim rows. */
 } fal_config;
 
 typedef struct fal_tensor_info {

@@ -42,20 +42,22 @@ __global__ void attn_bwd_pre_kernel(const bf16* __restrict__ ctx, const bf16* __
 }
 
 // ------------------------------------------------------------ fp32 debug path
+// Head h reads the key / value head g = h / (H / Hkv) (grouped-query attention).
 __global__ void attn_fwd_naive(const float* __restrict__ qkv, float* __restrict__ ctx, float* __restrict__ lse, int B,
-                               int T, int H, int hd, float scale) {
+                               int T, int H, int Hkv, int hd, float scale) {
   const long idx = blockIdx.x * (long)blockDim.x + threadIdx.x;
   if (idx >= (long)B * H * T) return;
   const int t = idx % T, h = (idx / T) % H, b = idx / ((long)T * H);
-  const int d = H * hd;
-  const long ld = 3L * d;
+  const int d = H * hd, g = h / (H / Hkv);
+  const long ld = (long)(H + 2 * Hkv) * hd;
+  const int kc = d + g * hd, vc = d + (Hkv + g) * hd;
   const float* q = qkv + ((long)b * T + t) * ld + h * hd;
   float o[128];
   for (int c = 0; c < hd; ++c) o[c] = 0.f;
   float m = -INFINITY, l = 0.f;
   for (int j = 0; j <= t; ++j) {
-    const float* k = qkv + ((long)b * T + j) * ld + d + h * hd;
-    const float* v = qkv + ((long)b * T + j) * ld + 2 * d + h * hd;
+    const float* k = qkv + ((long)b * T + j) * ld + kc;
+    const float* v = qkv + ((long)b * T + j) * ld + vc;
     float s = 0.f;
     for (int c = 0; c < hd; ++c) s = fmaf(q[c], k[c], s);
     s *= scale;
@@ -71,15 +73,17 @@ __global__ void attn_fwd_naive(const float* __restrict__ qkv, float* __restrict_
   lse[((long)b * H + h) * T + t] = (m + logf(l)) * LOG2E;
 }
 
-// Per query row: dq directly; dk, dv by fp32 atomics into dqkv (zeroed first).
+// Per query row: dq directly; dk, dv by fp32 atomics into dqkv (zeroed first),
+// which also sums them over the query heads of a key / value head's group.
 __global__ void attn_bwd_naive(const float* __restrict__ qkv, const float* __restrict__ ctx,
                                const float* __restrict__ lse, const float* __restrict__ dctx, float* __restrict__ dqkv,
-                               int B, int T, int H, int hd, float scale) {
+                               int B, int T, int H, int Hkv, int hd, float scale) {
   const long idx = blockIdx.x * (long)blockDim.x + threadIdx.x;
   if (idx >= (long)B * H * T) return;
   const int t = idx % T, h = (idx / T) % H, b = idx / ((long)T * H);
-  const int d = H * hd;
-  const long ld = 3L * d;
+  const int d = H * hd, g = h / (H / Hkv);
+  const long ld = (long)(H + 2 * Hkv) * hd;
+  const int kc = d + g * hd, vc = d + (Hkv + g) * hd;
   const float* q = qkv + ((long)b * T + t) * ld + h * hd;
   const float* o = ctx + ((long)b * T + t) * d + h * hd;
   const float* go = dctx + ((long)b * T + t) * d + h * hd;
@@ -89,14 +93,14 @@ __global__ void attn_bwd_naive(const float* __restrict__ qkv, const float* __res
   float dq[128];
   for (int c = 0; c < hd; ++c) dq[c] = 0.f;
   for (int j = 0; j <= t; ++j) {
-    const float* k = qkv + ((long)b * T + j) * ld + d + h * hd;
-    const float* v = qkv + ((long)b * T + j) * ld + 2 * d + h * hd;
+    const float* k = qkv + ((long)b * T + j) * ld + kc;
+    const float* v = qkv + ((long)b * T + j) * ld + vc;
     float s = 0.f, dp = 0.f;
     for (int c = 0; c < hd; ++c) { s = fmaf(q[c], k[c], s); dp = fmaf(go[c], v[c], dp); }
     const float p = expf(s * scale - L);
     const float ds = p * (dp - D);
-    float* dk = dqkv + ((long)b * T + j) * ld + d + h * hd;
-    float* dv = dqkv + ((long)b * T + j) * ld + 2 * d + h * hd;
+    float* dk = dqkv + ((long)b * T + j) * ld + kc;
+    float* dv = dqkv + ((long)b * T + j) * ld + vc;
     for (int c = 0; c < hd; ++c) {
       dq[c] = fmaf(ds, k[c], dq[c]);
       atomicAdd(dk + c, ds * q[c] * scale);
@@ -107,11 +111,12 @@ __global__ void attn_bwd_naive(const float* __restrict__ qkv, const float* __res
   for (int c = 0; c < hd; ++c) dqp[c] = dq[c] * scale;
 }
 
-__global__ void zero_kv_grad(float* dqkv, long rows, int d) {
-  const long n = rows * 2L * d;
+// Zeroes the key / value columns [d, d + dkv) of rows of width d + dkv.
+__global__ void zero_kv_grad(float* dqkv, long rows, int d, int dkv) {
+  const long n = rows * dkv;
   for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
-    const long r = i / (2L * d), c = i % (2L * d);
-    dqkv[r * 3L * d + d + c] = 0.f;
+    const long r = i / dkv, c = i % dkv;
+    dqkv[r * (long)(d + dkv) + d + c] = 0.f;
   }
 }
 
@@ -127,15 +132,17 @@ int check_launch(const char* what, std::string* msg) {
 }  // namespace
 
 int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
-             cudaStream_t s, std::string* msg) {
+             cudaStream_t s, std::string* msg, int Hkv) {
   if (B <= 0 || T <= 0) return 0;
+  if (Hkv <= 0) Hkv = H;
+  if (H % Hkv) { if (msg) *msg = "heads must be a multiple of the key/value heads"; return 1; }
   if (act_bf16) {
-    return attn_fwd_tc(B, T, H, hd, qkv, ctx, lse, dev_err, s, msg);
+    return attn_fwd_tc(B, T, H, Hkv, hd, qkv, ctx, lse, dev_err, s, msg);
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
     const long n = (long)B * H * T;
     attn_fwd_naive<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(reinterpret_cast<const float*>(qkv),
-                                                               reinterpret_cast<float*>(ctx), lse, B, T, H, hd,
+                                                               reinterpret_cast<float*>(ctx), lse, B, T, H, Hkv, hd,
                                                                1.f / sqrtf((float)hd));
   }
   count_launches(1);
@@ -144,8 +151,10 @@ int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* c
 
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
              const void* dctx, void* dqkv, float* dvec, int* dev_err, cudaStream_t s, std::string* msg,
-             int d_ready) {
+             int d_ready, int Hkv) {
   if (B <= 0 || T <= 0) return 0;
+  if (Hkv <= 0) Hkv = H;
+  if (H % Hkv) { if (msg) *msg = "heads must be a multiple of the key/value heads"; return 1; }
   const long rows = (long)B * T;
   const int d = H * hd;
   if (act_bf16) {
@@ -158,16 +167,17 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
           reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx), dvec, rows, T, H, hd);
       count_launches(1);
     }
-    const int r = attn_bwd2_tc(B, T, H, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
+    const int r = attn_bwd2_tc(B, T, H, Hkv, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
     if (r) return r;
     (void)d;
   } else {
     if (hd > 128) { if (msg) *msg = "fp32 attention needs head_dim <= 128"; return 6; }
-    zero_kv_grad<<<256, 256, 0, s>>>(reinterpret_cast<float*>(dqkv), rows, d);
+    zero_kv_grad<<<256, 256, 0, s>>>(reinterpret_cast<float*>(dqkv), rows, d, 2 * Hkv * hd);
     const long n = (long)B * H * T;
     attn_bwd_naive<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(
         reinterpret_cast<const float*>(qkv), reinterpret_cast<const float*>(ctx), lse,
-        reinterpret_cast<const float*>(dctx), reinterpret_cast<float*>(dqkv), B, T, H, hd, 1.f / sqrtf((float)hd));
+        reinterpret_cast<const float*>(dctx), reinterpret_cast<float*>(dqkv), B, T, H, Hkv, hd,
+        1.f / sqrtf((float)hd));
     count_launches(2);
   }
   return check_launch("attention backward", msg);

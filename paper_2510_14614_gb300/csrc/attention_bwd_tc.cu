@@ -46,12 +46,12 @@ constexpr int AB2_THREADS = 320;
 constexpr int AB2_STAGES = 4;
 
 struct AttnBwd2Params {
-  CUtensorMap qkv128, qkv64;  // [B*T, 3d] bf16, boxes 64 x 128 and 64 x 64, 128-byte swizzle
+  CUtensorMap qkv128, qkv64;  // [B*T, dq] bf16, dq = (H + 2 Hkv) hd, boxes 64 x 128 and 64 x 64, 128-byte swizzle
   CUtensorMap do128, do64;    // [B*T, d]  bf16, same boxes
   const float* lse;           // [B, H, T] log2 units of the scaled scores
   const float* dvec;          // [B, H, T] rowsum(dO * O)
-  bf16* dqkv;                 // [B*T, 3d]
-  int T, H, nblk;             // nblk: 128-row blocks per sequence
+  bf16* dqkv;                 // [B*T, dq]
+  int T, H, Hkv, nblk;        // Hkv key/value heads (each serves H / Hkv query heads); nblk: 128-row blocks
   float scale, scale_log2;
   int* err;
 };
@@ -93,18 +93,27 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
   // heaviest CTAs first: key block 0 (pass KV) / the last query block (pass Q)
   const int blk = KV ? bx : p.nblk - 1 - bx;
   const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
+  // Grouped-query attention: query head h uses key / value head g.  Pass KV
+  // runs one CTA per key / value head (on the grid row of the group's first
+  // query head) and streams the query blocks of every head of the group, so
+  // dK and dV sum over the group in TMEM.
+  const int gs = p.H / p.Hkv, g = h / gs;
+  if (KV && h % gs) return;
   const int d = p.H * HD;
+  const long dq = (long)(p.H + 2 * p.Hkv) * HD;    // qkv / dqkv row width
+  const int kcol = d + g * HD, vcol = d + (p.Hkv + g) * HD;
   const int row_base = b * p.T;
   const int r0 = blk * 128;  // first key (KV) or query (Q) row of this CTA
   const int nstream = (p.T + 63) / 64;
-  int j0, nit;
+  int j0, nit, nit_h;
   if (KV) {
     j0 = r0 / 64;             // query blocks that reach key r0 or later
-    nit = nstream - j0;
+    nit_h = nstream - j0;     // per query head of the group
+    nit = gs * nit_h;
   } else {
     j0 = 0;                   // key blocks up to the diagonal
     const int last = min(nstream - 1, (r0 + 127) / 64);
-    nit = last + 1;
+    nit = nit_h = last + 1;
   }
 
   if (threadIdx.x == 0) {
@@ -134,8 +143,8 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
       mbar_arrive_expect_tx(res_full, 2 * KCH * L::RES);
       for (int c = 0; c < KCH; ++c) {
         if (KV) {
-          tma_load_2d(base + L::RES_A + c * L::RES, &p.qkv128, d + h * HD + 64 * c, row_base + r0, res_full);
-          tma_load_2d(base + L::RES_B + c * L::RES, &p.qkv128, 2 * d + h * HD + 64 * c, row_base + r0, res_full);
+          tma_load_2d(base + L::RES_A + c * L::RES, &p.qkv128, kcol + 64 * c, row_base + r0, res_full);
+          tma_load_2d(base + L::RES_B + c * L::RES, &p.qkv128, vcol + 64 * c, row_base + r0, res_full);
         } else {
           tma_load_2d(base + L::RES_A + c * L::RES, &p.qkv128, h * HD + 64 * c, row_base + r0, res_full);
           tma_load_2d(base + L::RES_B + c * L::RES, &p.do128, h * HD + 64 * c, row_base + r0, res_full);
@@ -145,17 +154,18 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
     for (int it = 0; it < nit && ok; ++it) {
       const int s = it % AB2_STAGES;
       if (!mbar_wait(st_empty(s), ((it / AB2_STAGES) & 1) ^ 1u, abort_flag)) { ok = false; break; }
-      const int c0 = (j0 + it) * 64;  // first streamed row of this block
+      const int hq = KV ? g * gs + it / nit_h : h;     // query head of this streamed block
+      const int c0 = (j0 + it % nit_h) * 64;           // first streamed row of this block
       const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
       if (lane == 0) {
         mbar_arrive_expect_tx(st_full(s), L::STAGE);
         for (int c = 0; c < KCH; ++c) {
           if (KV) {
-            tma_load_2d(sb + c * L::STR, &p.qkv64, h * HD + 64 * c, row_base + c0, st_full(s));
-            tma_load_2d(sb + (KCH + c) * L::STR, &p.do64, h * HD + 64 * c, row_base + c0, st_full(s));
+            tma_load_2d(sb + c * L::STR, &p.qkv64, hq * HD + 64 * c, row_base + c0, st_full(s));
+            tma_load_2d(sb + (KCH + c) * L::STR, &p.do64, hq * HD + 64 * c, row_base + c0, st_full(s));
           } else {
-            tma_load_2d(sb + c * L::STR, &p.qkv64, d + h * HD + 64 * c, row_base + c0, st_full(s));
-            tma_load_2d(sb + (KCH + c) * L::STR, &p.qkv64, 2 * d + h * HD + 64 * c, row_base + c0, st_full(s));
+            tma_load_2d(sb + c * L::STR, &p.qkv64, kcol + 64 * c, row_base + c0, st_full(s));
+            tma_load_2d(sb + (KCH + c) * L::STR, &p.qkv64, vcol + 64 * c, row_base + c0, st_full(s));
           }
         }
       }
@@ -164,8 +174,9 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
         float* v = reinterpret_cast<float*>(sbase + L::VEC_OFF + s * 512);
         for (int i = lane; i < 64; i += 32) {
           const int t = c0 + i;
-          v[i] = t < p.T ? p.lse[(long)bh * p.T + t] : 0.f;
-          v[64 + i] = t < p.T ? p.dvec[(long)bh * p.T + t] : 0.f;
+          const long bq = (long)b * p.H + hq;
+          v[i] = t < p.T ? p.lse[bq * p.T + t] : 0.f;
+          v[64 + i] = t < p.T ? p.dvec[bq * p.T + t] : 0.f;
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(st_full(s));
@@ -253,7 +264,7 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
     bool ok = true;
     for (int it = 0; it < nit; ++it) {
       const int bb = it & 1, s = it % AB2_STAGES;
-      const int c0 = (j0 + it) * 64 + 32 * half;  // first streamed position of this warp's 32 columns
+      const int c0 = (j0 + it % nit_h) * 64 + 32 * half;  // first streamed position of this warp's 32 columns
       // sdp_full(it) also covers the accumulating MMAs of block it-2, the last
       // readers of the P / dS columns of buffer bb
       if (!mbar_wait(sdp_full(bb), (it >> 1) & 1, abort_flag)) { ok = false; break; }
@@ -302,8 +313,8 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
     // ------------------------------------------------ results: dK (scaled) and dV, or dQ (scaled)
     if (ok && mbar_wait(fin, 0, abort_flag)) {
       tc_fence_after();
-      bf16* out1 = p.dqkv + ((long)row_base + row) * 3L * d + (KV ? 2 * d : 0) + h * HD;  // dV or dQ
-      bf16* out2 = p.dqkv + ((long)row_base + row) * 3L * d + d + h * HD;               // dK
+      bf16* out1 = p.dqkv + ((long)row_base + row) * dq + (KV ? vcol : h * HD);  // dV or dQ
+      bf16* out2 = p.dqkv + ((long)row_base + row) * dq + kcol;                  // dK
       const float s1 = KV ? 1.f : p.scale;
 #pragma unroll
       for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
@@ -378,16 +389,17 @@ int launch_bwd2(const AttnBwd2Params& p, int BH, cudaStream_t s, std::string* ms
 
 }  // namespace
 
-int attn_bwd2_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-                 void* dqkv, int* dev_err, cudaStream_t s, std::string* msg) {
+int attn_bwd2_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
+                 const float* dvec, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
   if (hd != 64 && hd != 128) { if (msg) *msg = "tcgen05 attention needs head_dim 64 or 128"; return 6; }
+  if (Hkv <= 0 || H % Hkv) { if (msg) *msg = "heads must be a multiple of the key/value heads"; return 1; }
   AttnBwd2Params p;
   memset(&p, 0, sizeof(p));
-  const long d = (long)H * hd;
+  const long d = (long)H * hd, dq = (long)(H + 2 * Hkv) * hd;
   const unsigned long long rows = (unsigned long long)B * T;
-  if (!tma_map_2d(&p.qkv128, qkv, 0, 3 * d, rows, 3 * d, 64, 128, 1, msg) ||
-      !tma_map_2d(&p.qkv64, qkv, 0, 3 * d, rows, 3 * d, 64, 64, 1, msg) ||
+  if (!tma_map_2d(&p.qkv128, qkv, 0, dq, rows, dq, 64, 128, 1, msg) ||
+      !tma_map_2d(&p.qkv64, qkv, 0, dq, rows, dq, 64, 64, 1, msg) ||
       !tma_map_2d(&p.do128, dctx, 0, d, rows, d, 64, 128, 1, msg) ||
       !tma_map_2d(&p.do64, dctx, 0, d, rows, d, 64, 64, 1, msg))
     return 1;
@@ -396,6 +408,7 @@ int attn_bwd2_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx,
   p.dqkv = reinterpret_cast<bf16*>(dqkv);
   p.T = T;
   p.H = H;
+  p.Hkv = Hkv;
   p.nblk = (T + 127) / 128;
   p.scale = 1.f / sqrtf((float)hd);
   p.scale_log2 = 1.4426950408889634f / sqrtf((float)hd);

@@ -36,10 +36,10 @@ constexpr int AT_BM = 128, AT_BN = 128;
 constexpr float AT_RESCALE_LOG2 = 8.f;  // raise the exponent's maximum only beyond 2^8 growth
 
 struct AttnParams {
-  CUtensorMap qkv;  // [B*T rows, 3*H*hd cols] bf16, box 64 x 128, 128-byte swizzle
+  CUtensorMap qkv;  // [B*T rows, (H + 2 Hkv)*hd cols] bf16, box 64 x 128, 128-byte swizzle
   bf16* ctx;
   float* lse;
-  int T, H, nq;
+  int T, H, Hkv, nq;  // Hkv key/value heads, each serving H / Hkv query heads (Hkv = H: MHA)
   float scale_log2;
   int* err;
 };
@@ -91,6 +91,8 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
   const int t2 = p.nq - 1 - (int)blockIdx.x;  // heaviest 256-query blocks first
   const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
   const int d = p.H * HD;
+  const int g = h / (p.H / p.Hkv);                     // key / value head of this query head
+  const int kcol = d + g * HD, vcol = d + (p.Hkv + g) * HD;
   const int row_base = b * p.T;
   const int nkb_all = (p.T + AT_BN - 1) / AT_BN;
   // causal: tile A sees key blocks 0..2t2, tile B 0..2t2+1 (none if it starts past T)
@@ -132,7 +134,7 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
       if (lane == 0) {
         mbar_arrive_expect_tx(kfull(s), KCH * L::CHUNK);
         for (int c = 0; c < KCH; ++c)
-          tma_load_2d(base + L::K_OFF + (s * KCH + c) * L::CHUNK, &p.qkv, d + h * HD + 64 * c, row_base + j * AT_BN,
+          tma_load_2d(base + L::K_OFF + (s * KCH + c) * L::CHUNK, &p.qkv, kcol + 64 * c, row_base + j * AT_BN,
                       kfull(s));
       }
       __syncwarp();
@@ -140,7 +142,7 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
       if (lane == 0) {
         mbar_arrive_expect_tx(vfull(s), KCH * L::CHUNK);
         for (int c = 0; c < KCH; ++c)
-          tma_load_2d(base + L::V_OFF + (s * KCH + c) * L::CHUNK, &p.qkv, 2 * d + h * HD + 64 * c,
+          tma_load_2d(base + L::V_OFF + (s * KCH + c) * L::CHUNK, &p.qkv, vcol + 64 * c,
                       row_base + j * AT_BN, vfull(s));
       }
       __syncwarp();
@@ -335,7 +337,7 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
 }
 
 template <int HD>
-int launch_fwd_tc(int B, int T, int H, const void* qkv, void* ctx, float* lse, int* err, cudaStream_t s,
+int launch_fwd_tc(int B, int T, int H, int Hkv, const void* qkv, void* ctx, float* lse, int* err, cudaStream_t s,
                   std::string* msg) {
   using L = Attn2Smem<HD>;
   static bool set = false;
@@ -349,12 +351,13 @@ int launch_fwd_tc(int B, int T, int H, const void* qkv, void* ctx, float* lse, i
   }
   AttnParams p;
   memset(&p, 0, sizeof(p));
-  const long d = (long)H * HD;
-  if (!tma_map_2d(&p.qkv, qkv, 0, 3 * d, (unsigned long long)B * T, 3 * d, 64, AT_BM, 1, msg)) return 1;
+  const long dq = (long)(H + 2 * Hkv) * HD;
+  if (!tma_map_2d(&p.qkv, qkv, 0, dq, (unsigned long long)B * T, dq, 64, AT_BM, 1, msg)) return 1;
   p.ctx = reinterpret_cast<bf16*>(ctx);
   p.lse = lse;
   p.T = T;
   p.H = H;
+  p.Hkv = Hkv;
   p.nq = (T + 255) / 256;  // 256-query blocks
   p.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
   p.err = err;
@@ -366,12 +369,13 @@ int launch_fwd_tc(int B, int T, int H, const void* qkv, void* ctx, float* lse, i
 
 }  // namespace
 
-int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
-                std::string* msg) {
+int attn_fwd_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
+                cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
+  if (Hkv <= 0 || H % Hkv) { if (msg) *msg = "heads must be a multiple of the key/value heads"; return 1; }
   int r;
-  if (hd == 64) r = launch_fwd_tc<64>(B, T, H, qkv, ctx, lse, dev_err, s, msg);
-  else if (hd == 128) r = launch_fwd_tc<128>(B, T, H, qkv, ctx, lse, dev_err, s, msg);
+  if (hd == 64) r = launch_fwd_tc<64>(B, T, H, Hkv, qkv, ctx, lse, dev_err, s, msg);
+  else if (hd == 128) r = launch_fwd_tc<128>(B, T, H, Hkv, qkv, ctx, lse, dev_err, s, msg);
   else { if (msg) *msg = "tcgen05 attention needs head_dim 64 or 128"; return 6; }
   if (r) return r;
   cudaError_t e = cudaGetLastError();

@@ -74,13 +74,15 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
 // ctx: activation [B*T, H*hd]; lse: fp32 [B, H, T] in log2 units of the scaled scores.
 // bf16: tcgen05 kernel (dev_err receives DEV_ERR_TIMEOUT if a bounded wait expires);
 // fp32 debug: one thread per query row.
+// Hkv: key/value heads (grouped-query attention, qkv rows of (H + 2 Hkv) * hd);
+// 0 means H (multi-head attention).
 int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
-             cudaStream_t s, std::string* msg);
+             cudaStream_t s, std::string* msg, int Hkv = 0);
 // dvec: fp32 [B, H, T] scratch (receives D = rowsum(dO * O)); d_ready: dvec
 // already holds D (computed by the GEMM that produced dctx).
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
              const float* lse, const void* dctx, void* dqkv, float* dvec, int* dev_err,
-             cudaStream_t s, std::string* msg, int d_ready = 0);
+             cudaStream_t s, std::string* msg, int d_ready = 0, int Hkv = 0);
 
 // ---------------------------------------------------------------- elementwise
 struct LnFwdArgs {
@@ -179,13 +181,15 @@ int num_sms();
 bool tma_map_2d(void* map128, const void* ptr, int f32, unsigned long long inner, unsigned long long outer,
                 unsigned long long ld, unsigned box_inner, unsigned box_outer, int swizzle128, std::string* msg);
 
-// tcgen05 flash-attention forward (bf16, head_dim 64 or 128).
-int attn_fwd_tc(int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err, cudaStream_t s,
-                std::string* msg);
+// tcgen05 flash-attention forward (bf16, head_dim 64 or 128); Hkv key/value
+// heads, each serving H / Hkv query heads (grouped-query attention; Hkv = H:
+// multi-head attention), qkv rows of (H + 2 Hkv) * hd.
+int attn_fwd_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
+                cudaStream_t s, std::string* msg);
 // Two-pass tcgen05 attention backward (dK/dV per key block, then dQ per query
 // block, all accumulated in TMEM; no dQ accumulator).  dvec = rowsum(dO * O).
-int attn_bwd2_tc(int B, int T, int H, int hd, const void* qkv, const void* dctx, const float* lse, const float* dvec,
-                 void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
+int attn_bwd2_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
+                 const float* dvec, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
 
 // Process-wide count of kernel launches made by the library.
 void count_launches(long long n);

@@ -77,6 +77,7 @@ struct fal_handle {
   int bf = 1;          // activations bf16 (else fp32 debug)
   size_t asz = 2;      // activation element size
   int B = 0, T = 0, d = 0, H = 0, hd = 0, F = 0, L = 0, V = 0, Vp = 0;
+  int Hkv = 0, DQ = 0;  // key/value heads (GQA groups) and the fused QKV width d + 2 Hkv hd
   long BT = 0;
   cudaStream_t sm = nullptr, ss = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr, ev_mid = nullptr;
@@ -166,8 +167,8 @@ void build_table(fal_handle* h) {
     const std::string p = "h" + std::to_string(i) + ".";
     add_tensor(h, nodec, nodec, p + "ln1.g", d, 0, 0);
     add_tensor(h, nodec, nodec, p + "ln1.b", d, 0, 0);
-    add_tensor(h, dec, nodec, p + "attn.w_qkv", 3 * d, d, 1);
-    add_tensor(h, dec, nodec, p + "attn.b_qkv", 3 * d, 0, 0);
+    add_tensor(h, dec, nodec, p + "attn.w_qkv", h->DQ, d, 1);
+    add_tensor(h, dec, nodec, p + "attn.b_qkv", h->DQ, 0, 0);
     add_tensor(h, dec, nodec, p + "attn.w_o", d, d, 1);
     add_tensor(h, dec, nodec, p + "attn.b_o", d, 0, 0);
     if (var == FAL_GPT || var == FAL_FALPLUS || (var == FAL_ABLATION2 && i == 0)) {
@@ -257,6 +258,10 @@ int validate(const fal_config* c, std::string* msg) {
     return FAL_ERR_ARG;
   }
   if (!(c->clip_norm >= 0.f)) { *msg = "clip_norm must be >= 0"; return FAL_ERR_ARG; }
+  if (c->kv_heads < 0 || (c->kv_heads > 0 && c->heads % c->kv_heads)) {
+    *msg = "kv_heads must be 0 (one per head) or divide heads";
+    return FAL_ERR_ARG;
+  }
   if (c->precision != FAL_BF16 && c->precision != FAL_FP32_DEBUG) { *msg = "bad precision"; return FAL_ERR_ARG; }
   if (c->schedule != FAL_SCHED_SERIAL && c->schedule != FAL_SCHED_TWO_STREAM) { *msg = "bad schedule"; return FAL_ERR_ARG; }
   const int hd = c->d_model / c->heads;
@@ -281,6 +286,8 @@ void init_dims(fal_handle* h, const fal_config* c) {
   h->Vp = (c->vocab + 63) / 64 * 64;
   h->BT = (long)h->B * h->T;
   h->reuse = c->reuse_layer > 1 ? c->reuse_layer - 1 : 0;
+  h->Hkv = c->kv_heads > 0 ? c->kv_heads : h->H;
+  h->DQ = h->d + 2 * h->Hkv * h->hd;
 }
 
 // MLP-input rule of block i (the block equations of each variant).
@@ -326,7 +333,7 @@ void carve(fal_handle* h, uint8_t* base) {
     A.ln1_rstd = b.take<float>(BT);
     A.u = b.take<uint8_t>(BT * d * a);
     A.m = b.take<uint8_t>(BT * d * a);
-    A.qkv = b.take<uint8_t>(BT * 3 * d * a);
+    A.qkv = b.take<uint8_t>(BT * h->DQ * a);
     A.ctx = b.take<uint8_t>(BT * d * a);
     A.lse = b.take<float>((size_t)h->B * h->H * h->T);
     A.h = b.take<uint8_t>(BT * F * a);
@@ -364,9 +371,9 @@ void carve(fal_handle* h, uint8_t* base) {
   h->dA_act = b.take<uint8_t>(BT * d * a);
   h->dctx = b.take<uint8_t>(BT * d * a);
   h->dh = b.take<uint8_t>(BT * F * a);
-  h->dqkv = b.take<uint8_t>(BT * 3 * d * a);
+  h->dqkv = b.take<uint8_t>(BT * h->DQ * a);
   h->dvec = b.take<float>((size_t)h->B * h->H * h->T);
-  const int cs_cols = 3 * h->d > h->F ? 3 * h->d : h->F;  // widest column reduction: b_qkv or b_up
+  const int cs_cols = h->DQ > h->F ? h->DQ : h->F;  // widest column reduction: b_qkv or b_up
   h->part0 = b.take<float>(colsum_partial_floats(cs_cols));
   h->part1 = b.take<float>(colsum_partial_floats(cs_cols));
   h->gn_part = b.take<float>(grad_norm_partials());
@@ -555,9 +562,9 @@ void qkv_and_attention(Ctx& c, int i, cudaStream_t s, cudaStream_t after_qkv = n
   LayerA& A = h->la[i];
   const LayerP& p = h->lp[i];
   const int BT = (int)h->BT, d = h->d;
-  EpiParams e = epi_out(A.qkv, 3L * d, OUT_ACT);
+  EpiParams e = epi_out(A.qkv, h->DQ, OUT_ACT);
   e.bias = Pp(h, p.b_qkv);
-  gemm(c, call1(BT, 3 * d, seg(A.u, d, 0, Wp(h, p.w_qkv), d, 0, d), e), s, "QKV projection");
+  gemm(c, call1(BT, h->DQ, seg(A.u, d, 0, Wp(h, p.w_qkv), d, 0, d), e), s, "QKV projection");
   if (after_qkv) {
     // the other stream's work starts behind the projection, beside the attention
     cudaEventRecord(h->ev_mid, s);
@@ -566,7 +573,8 @@ void qkv_and_attention(Ctx& c, int i, cudaStream_t s, cudaStream_t after_qkv = n
   if (!c.ok()) return;
   h->err.clear();
   ProfScope ps(h, s, 1, attn_fwd_flops(h), "attention forward");
-  c.check(attn_fwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dev_err, s, &h->err), "attention forward");
+  c.check(attn_fwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dev_err, s, &h->err, h->Hkv),
+          "attention forward");
 }
 
 void up_gemm(Ctx& c, int i, cudaStream_t s) {
@@ -767,13 +775,13 @@ void attn_backward(Ctx& c, int i, const float* da, const void* da_act, cudaStrea
   {
     ProfScope ps(h, s, 2, 2.0 * attn_fwd_flops(h), "attention backward");
     c.check(attn_bwd(h->bf, h->B, h->T, h->H, h->hd, A.qkv, A.ctx, A.lse, h->dctx, h->dqkv, h->dvec,
-                     h->dev_err, s, &h->err, d_ready ? 1 : 0),
+                     h->dev_err, s, &h->err, d_ready ? 1 : 0, h->Hkv),
             "attention backward");
   }
-  gemm(c, group_calls({call1(3 * d, d, wgrad_seg(h, h->dqkv, 3 * d, A.u, d), wgrad_out(h, p.w_qkv, d)),
-                       call1(BT, d, dgrad_seg(h, h->dqkv, 3 * d, p.w_qkv, d), epi_out(h->dU, d, OUT_F32))}),
+  gemm(c, group_calls({call1(h->DQ, d, wgrad_seg(h, h->dqkv, h->DQ, A.u, d), wgrad_out(h, p.w_qkv, d)),
+                       call1(BT, d, dgrad_seg(h, h->dqkv, h->DQ, p.w_qkv, d), epi_out(h->dU, d, OUT_F32))}),
        s, "QKV wgrad + dgrad");
-  colsum_(c, s, part, h->dqkv, 1, 3L * d, 3 * d, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_qkv),
+  colsum_(c, s, part, h->dqkv, 1, h->DQ, h->DQ, nullptr, 0, nullptr, nullptr, nullptr, nullptr, nullptr, Gp(h, p.b_qkv),
           nullptr, 0);
 }
 
@@ -1229,7 +1237,7 @@ int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n
   else if (nm == "u") { if (lay) src = h->la[layer].u; }
   else if (nm == "m") { if (lay) src = mlp_in(h, layer); }
   else if (nm == "ctx") { if (lay) src = h->la[layer].ctx; }
-  else if (nm == "qkv") { if (lay) src = h->la[layer].qkv; cols = 3 * d; ld = 3L * d; }
+  else if (nm == "qkv") { if (lay) src = h->la[layer].qkv; cols = h->DQ; ld = h->DQ; }
   else if (nm == "h") { if (lay) src = h->la[layer].h; cols = F; ld = F; }
   else if (nm == "g") { if (lay) src = h->la[layer].g; cols = F; ld = F; }
   else if (nm == "a1") { src = h->a1; is_act = 0; }

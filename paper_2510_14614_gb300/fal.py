@@ -26,7 +26,7 @@ class FalConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("variant", "layers", "d_model", "heads", "d_ff", "seq", "batch", "vocab",
                                             "precision", "schedule")] + \
                [(n, ctypes.c_float) for n in ("lr", "beta1", "beta2", "eps", "weight_decay")] + \
-               [("reuse_layer", ctypes.c_int), ("clip_norm", ctypes.c_float)]
+               [("reuse_layer", ctypes.c_int), ("clip_norm", ctypes.c_float), ("kv_heads", ctypes.c_int)]
 
 
 class FalTensorInfo(ctypes.Structure):
@@ -125,9 +125,10 @@ def _stream_ptr(s):
 
 
 def make_config(variant, layers, d_model, heads, d_ff, seq, batch, vocab, precision="bf16", schedule="serial",
-                lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=1e-3, reuse_layer=1, clip_norm=0.0):
+                lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=1e-3, reuse_layer=1, clip_norm=0.0,
+                kv_heads=0):
     return FalConfig(VARIANT[variant], layers, d_model, heads, d_ff, seq, batch, vocab, PRECISION[precision],
-                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay, reuse_layer, clip_norm)
+                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay, reuse_layer, clip_norm, kv_heads)
 
 
 def workspace_size(cfg: FalConfig) -> int:
@@ -300,7 +301,9 @@ class Model:
     def tap(self, name, layer=0):
         c = self.cfg
         bt = c.batch * c.seq
-        cols = {"qkv": 3 * c.d_model, "h": c.d_ff, "g": c.d_ff, "logits": c.vocab}.get(name, c.d_model)
+        kv = c.kv_heads or c.heads
+        dq = c.d_model + 2 * kv * (c.d_model // c.heads)
+        cols = {"qkv": dq, "h": c.d_ff, "g": c.d_ff, "logits": c.vocab}.get(name, c.d_model)
         out = np.empty((bt, cols), np.float32)
         _check(lib().fal_get_tap(self.h, name.encode(), layer, out.ctypes.data_as(ctypes.c_void_p), out.size),
                self.h, f"fal_get_tap({name})")

@@ -20,7 +20,7 @@ def _model(variant, s, schedule="serial", **overrides):
     from paper_2510_14614_gb300 import fal
     hp = dict(synth.adamw_hparams(), **overrides)
     cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
-                          precision=s.precision, schedule=schedule, **hp)
+                          precision=s.precision, schedule=schedule, kv_heads=s.kv_heads, **hp)
     return fal.Model(cfg)
 
 
@@ -361,3 +361,20 @@ def test_prefill_last_logits_match_oracle(variant, shape, schedule):
     assert e.value.code == fal.FAL_ERR_STATE
     # a training step after the prefill still works
     assert np.isfinite(m.train_step(tok, tgt))
+
+
+# Grouped-query attention (App. E): key/value heads shared by groups of query
+# heads; 4 query heads of 64 in 2 groups, and of 128 in 1 group (MQA).
+GQA_S = synth.Shape("gqa_ragged", 3, 256, 4, 512, 130, 2, 777, "bf16", kv_heads=2)
+GQA_HD128 = synth.Shape("gqa_hd128", 2, 512, 4, 1024, 200, 1, 999, "bf16", kv_heads=1)
+
+
+@pytest.mark.parametrize("variant,schedule", [("fal", "two_stream"), ("gpt", "serial"), ("falplus", "serial")])
+@pytest.mark.parametrize("s", [GQA_S, GQA_HD128], ids=lambda s: s.name)
+def test_gqa_bf16_parity(variant, schedule, s):
+    _check_parity(variant, s, 1e-2, schedule=schedule)
+
+
+@pytest.mark.parametrize("variant", ["fal", "gpt"])
+def test_gqa_fp32_debug_parity(variant):
+    _check_parity(variant, synth.SHAPES["tiny"].replace(layers=3, kv_heads=2), 1e-4)
