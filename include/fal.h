@@ -6,7 +6,8 @@
  *   GPT  (Eq. 1, Sec. 2):   X_{i+1} = X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i + MHA_i(LN(X_i))))
  *   FAL  (Eq. 2, Sec. 4.1): X_{i+1} = X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i) + LN_F(MHA_1(LN(X_1))))
  *        LN(X_i) is the same LayerNorm output that feeds MHA_i; LN_F is one
- *        LayerNorm shared by all blocks (applied "only once", Sec. 4.1).
+ *        LayerNorm shared by all blocks (the first attention output is normalised
+ *        a single time, Sec. 4.1).
  *   FAL+ (Sec. 5, App. D.1): block 1 is the standard block; block i >= 2 feeds
  *        MLP_i(LN(X_i + MHA_i(LN(X_i))) + LN_{F,i}(MHA_1(LN(X_1)))).
  * The paper's comparison blocks, built from the same kernels:
@@ -122,8 +123,8 @@ void fal_destroy(fal_handle* h);
  * reported as FAL_ERR_ARG at the next synchronizing call. */
 int fal_forward(fal_handle* h, const int32_t* tokens, const int32_t* targets, float* loss_host);
 
-/* Forward-only pass for inference, the paper's "forward step time without
- * gradient calculation" that matches the time to first token (App. E): the
+/* Forward-only pass for inference: App. E times the forward step without
+ * gradients as the time to first token.  Runs the
  * stack over tokens [B, T] (int32 row-major, device or host), the final
  * LayerNorm, and the tied LM head for the last position of every sequence
  * only.  last_logits: fp32 [B, V] row-major, device or host, or NULL to leave

@@ -12,8 +12,8 @@ NumPy (matmul is the only library primitive used):
   * FAL block, Eq. 2 (Sec. 4.1), every block i including the first:
         X_{i+1} = X_i + MHA_i(LN(X_i)) + MLP_i(LN(X_i) + LN(MHA_1(LN(X_1))))
     with LN(X_i) the same LayerNorm output that feeds MHA_i, and one LayerNorm
-    LN_F on the first attention output shared by all blocks (Sec. 4.1: "apply
-    LN to the first attention output only once").
+    LN_F on the first attention output shared by all blocks (Sec. 4.1: the
+    first attention output is normalised a single time).
   * FAL+ block (Sec. 5; App. D.1 equation): block 1 is the standard block;
     block i >= 2 feeds MLP_i(LN(X_i + MHA_i(LN(X_i))) + LN_{F,i}(MHA_1(LN(X_1))))
     with its own LayerNorm LN_{F,i} on the first attention output.
