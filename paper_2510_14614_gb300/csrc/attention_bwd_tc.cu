@@ -151,11 +151,12 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
         }
       }
     }
-    for (int it = 0; it < nit && ok; ++it) {
+    // (jj, hq): streamed block index within its query head, and that head
+    // (pass KV walks the heads of the group one after another)
+    for (int it = 0, jj = 0, hq = KV ? g * gs : h; it < nit && ok; ++it) {
       const int s = it % AB2_STAGES;
       if (!mbar_wait(st_empty(s), ((it / AB2_STAGES) & 1) ^ 1u, abort_flag)) { ok = false; break; }
-      const int hq = KV ? g * gs + it / nit_h : h;     // query head of this streamed block
-      const int c0 = (j0 + it % nit_h) * 64;           // first streamed row of this block
+      const int c0 = (j0 + jj) * 64;                   // first streamed row of this block
       const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
       if (lane == 0) {
         mbar_arrive_expect_tx(st_full(s), L::STAGE);
@@ -182,6 +183,7 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
         if (lane == 0) mbar_arrive(st_full(s));
       }
       __syncwarp();
+      if (++jj == nit_h) { jj = 0; ++hq; }
     }
     if (!ok && lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
   } else if (warp == 1) {
@@ -262,9 +264,10 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
       d_r = p.dvec[(long)bh * p.T + row];
     }
     bool ok = true;
-    for (int it = 0; it < nit; ++it) {
+    for (int it = 0, jj = -1; it < nit; ++it) {
+      if (++jj == nit_h) jj = 0;  // streamed block index within its query head
       const int bb = it & 1, s = it % AB2_STAGES;
-      const int c0 = (j0 + it % nit_h) * 64 + 32 * half;  // first streamed position of this warp's 32 columns
+      const int c0 = (j0 + jj) * 64 + 32 * half;  // first streamed position of this warp's 32 columns
       // sdp_full(it) also covers the accumulating MMAs of block it-2, the last
       // readers of the P / dS columns of buffer bb
       if (!mbar_wait(sdp_full(bb), (it >> 1) & 1, abort_flag)) { ok = false; break; }
