@@ -1,6 +1,6 @@
 // Row-streaming LayerNorm forward and backward: the LN_1, LN_2, LN_F and final
 // LayerNorms of the blocks (Eq. 1, Eq. 2) with their backward, for rows of up
-// to 2048 features.
+// to 4096 features.
 //
 // These kernels are bound by HBM bandwidth.  Warp-per-row kernels that load a
 // row into registers keep too few bytes in flight per SM (every load holds an
@@ -9,7 +9,7 @@
 // (cp.async.bulk, issued by one producer thread, completion counted on an
 // mbarrier), so several rows per SM are always on their way from HBM without
 // holding registers.  Eight consumer warps share each row: every thread owns
-// up to two 4-column groups of it, row statistics are reduced with warp
+// up to four 4-column groups of it, row statistics are reduced with warp
 // shuffles and one named barrier, and each row's outputs leave with coalesced
 // 16-byte stores.  The backward also accumulates the affine parameters'
 // gradient column sums in registers across all rows of the CTA, so no second
@@ -35,11 +35,16 @@ constexpr float LR_EPS = 1e-5f;
 constexpr int LR_WARPS = 8;                 // consumer warps
 constexpr int LR_CONS = LR_WARPS * 32;      // consumer threads
 constexpr int LR_THREADS = LR_CONS + 32;    // + one producer warp
-constexpr int LR_MAX_D = 2 * 4 * LR_CONS;   // two 4-column groups per consumer thread
+constexpr int LR_MAX_D = 4 * 4 * LR_CONS;   // up to four 4-column groups per consumer thread
 constexpr int LR_MAX_STAGES = 8;
-constexpr uint32_t LR_STAGE_BUDGET = 96 * 1024;  // two CTAs per SM
+constexpr uint32_t LR_STAGE_BUDGET = 96 * 1024;  // two CTAs per SM (rows of up to 2048 features)
+constexpr uint32_t LR_WIDE_BUDGET = 192 * 1024;  // one CTA per SM (wider rows: four column groups)
 constexpr uint32_t LR_TAIL_BYTES = 16 * LR_MAX_STAGES + 32 * 4 + 16;  // barriers, reduction slots, abort flag
 constexpr uint32_t LR_SMEM_MAX = LR_STAGE_BUDGET + LR_TAIL_BYTES;
+constexpr uint32_t LR_WIDE_SMEM_MAX = LR_WIDE_BUDGET + LR_TAIL_BYTES;
+// Column groups per consumer thread for rows of d features, and CTAs per SM.
+__host__ __device__ constexpr int lr_nch(int d) { return d <= 4 * LR_CONS ? 1 : d <= 8 * LR_CONS ? 2 : 4; }
+__host__ __device__ constexpr int lr_ctas_per_sm(int nch) { return nch > 2 ? 1 : 2; }
 
 // fp32 row-major [rows, d] inputs copied into each stage, in slot order.
 struct RowSrc {
@@ -118,7 +123,7 @@ __device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 
 
 // y = LN(x) (* gamma + beta); optional fp32 copy; out2 = y + add_src * add_g + add_b.
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes,
+__global__ void __launch_bounds__(LR_THREADS, lr_ctas_per_sm(NCH)) ln_fwd_rows_kernel(const LnFwdArgs a, int stages, uint32_t stage_bytes,
                                                                     long long wait_ns, int stall_rows) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
@@ -212,7 +217,7 @@ __global__ void __launch_bounds__(LR_THREADS, 2) ln_fwd_rows_kernel(const LnFwdA
 // dx = rstd * (g - mean(g) - xhat * mean(g * xhat)) + dres with g = (dy + dy2) * gamma;
 // optional per-CTA column sums of (dy + dy2) * xhat and (dy + dy2).
 template <typename act_t, int NCH>
-__global__ void __launch_bounds__(LR_THREADS, 2) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes,
+__global__ void __launch_bounds__(LR_THREADS, lr_ctas_per_sm(NCH)) ln_bwd_rows_kernel(const LnBwdArgs a, int stages, uint32_t stage_bytes,
                                                                     long long wait_ns, int stall_rows) {
   extern __shared__ __align__(16) uint8_t smem[];
   float* red;
@@ -315,55 +320,62 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 
 // Stage count for `nin` input rows of d floats, 0 when fewer than two fit.
 int ring_stages(int nin, int d, uint32_t* stage_bytes) {
   *stage_bytes = (uint32_t)nin * (uint32_t)d * 4u;
-  int st = (int)(LR_STAGE_BUDGET / *stage_bytes);
+  const uint32_t budget = lr_nch(d) > 2 ? LR_WIDE_BUDGET : LR_STAGE_BUDGET;
+  int st = (int)(budget / *stage_bytes);
   if (st > LR_MAX_STAGES) st = LR_MAX_STAGES;
   return st >= 2 ? st : 0;
 }
 
 template <typename K>
-bool set_smem_attr(K kernel) {
-  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LR_SMEM_MAX) == cudaSuccess;
+bool set_smem_attr(K kernel, uint32_t bytes = LR_SMEM_MAX) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) == cudaSuccess;
 }
 
 std::atomic<int> g_stall_rows{-1};
 std::atomic<long long> g_wait_ns{0};
 
-int rows_grid(int rows) {
-  int g = 2 * num_sms();
+int rows_grid(int rows, int d) {
+  int g = lr_ctas_per_sm(lr_nch(d)) * num_sms();
   if (g > kMaxColsumChunks) g = kMaxColsumChunks;  // per-CTA column partials must fit colsum_partial_floats(d)
   return rows < g ? rows : g;
 }
 
 template <typename act_t>
 int ln_fwd_rows(const LnFwdArgs& a, cudaStream_t s) {
-  static const bool attr = set_smem_attr(ln_fwd_rows_kernel<act_t, 1>) && set_smem_attr(ln_fwd_rows_kernel<act_t, 2>);
+  static const bool attr = set_smem_attr(ln_fwd_rows_kernel<act_t, 1>) && set_smem_attr(ln_fwd_rows_kernel<act_t, 2>) &&
+                           set_smem_attr(ln_fwd_rows_kernel<act_t, 4>, LR_WIDE_SMEM_MAX);
   if (!attr) return 1;
   const bool has2 = a.out2 != nullptr && a.add_src != nullptr;
   uint32_t sb;
   const int st = ring_stages(has2 ? 2 : 1, a.d, &sb);
   if (!st) return 1;
   const uint32_t smem = (uint32_t)st * sb + LR_TAIL_BYTES;
-  const int grid = rows_grid(a.rows);
+  const int grid = rows_grid(a.rows, a.d);
   const long long w = g_wait_ns.load();
   const int sr = g_stall_rows.load();
-  if (a.d <= 4 * LR_CONS) ln_fwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
-  else ln_fwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  const int nch = lr_nch(a.d);
+  if (nch == 1) ln_fwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else if (nch == 2) ln_fwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else ln_fwd_rows_kernel<act_t, 4><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
   return 0;
 }
 
 template <typename act_t>
 int ln_bwd_rows(const LnBwdArgs& a, cudaStream_t s) {
-  static const bool attr = set_smem_attr(ln_bwd_rows_kernel<act_t, 1>) && set_smem_attr(ln_bwd_rows_kernel<act_t, 2>);
+  static const bool attr = set_smem_attr(ln_bwd_rows_kernel<act_t, 1>) && set_smem_attr(ln_bwd_rows_kernel<act_t, 2>) &&
+                           set_smem_attr(ln_bwd_rows_kernel<act_t, 4>, LR_WIDE_SMEM_MAX);
   if (!attr) return 1;
   uint32_t sb;
   const int st = ring_stages(2 + (a.dy2 ? 1 : 0) + (a.dres ? 1 : 0), a.d, &sb);
   if (!st) return 1;
   const uint32_t smem = (uint32_t)st * sb + LR_TAIL_BYTES;
-  const int grid = rows_grid(a.rows);
+  const int grid = rows_grid(a.rows, a.d);
   const long long w = g_wait_ns.load();
   const int sr = g_stall_rows.load();
-  if (a.d <= 4 * LR_CONS) ln_bwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
-  else ln_bwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  const int nch = lr_nch(a.d);
+  if (nch == 1) ln_bwd_rows_kernel<act_t, 1><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else if (nch == 2) ln_bwd_rows_kernel<act_t, 2><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
+  else ln_bwd_rows_kernel<act_t, 4><<<grid, LR_THREADS, smem, s>>>(a, st, sb, w, sr);
   return 0;
 }
 
@@ -384,7 +396,7 @@ int ln_bwd_bulk(int act_bf16, const LnBwdArgs& a, cudaStream_t s) {
   if (r) return r;
   if (a.cs_part) {
     const bool sum_dx = a.dxs_out || a.dxs_out2;
-    return colsum_finish(a.cs_part, rows_grid(a.rows), a.d, a.cs_out1, a.cs_out0, nullptr, a.cs_accumulate, s,
+    return colsum_finish(a.cs_part, rows_grid(a.rows, a.d), a.d, a.cs_out1, a.cs_out0, nullptr, a.cs_accumulate, s,
                          sum_dx ? 3 : 2, a.dxs_out, a.dxs_out2);
   }
   return 0;

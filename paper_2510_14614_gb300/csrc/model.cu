@@ -272,7 +272,7 @@ int validate(const fal_config* c, std::string* msg) {
     if (hd > 128) { *msg = "fp32 debug path needs head_dim <= 128"; return FAL_ERR_ARG; }
     if (c->d_model % 4 || c->d_ff % 4) { *msg = "d_model and d_ff must be multiples of 4"; return FAL_ERR_ARG; }
   }
-  if (c->d_model > 2048) { *msg = "d_model above 2048 is not supported by the LayerNorm kernels"; return FAL_ERR_ARG; }
+  if (c->d_model > 4096) { *msg = "d_model above 4096 is not supported by the LayerNorm kernels"; return FAL_ERR_ARG; }
   if ((long)c->batch * c->seq > 65535) { *msg = "batch*seq above 65535 is not supported"; return FAL_ERR_ARG; }
   return FAL_OK;
 }

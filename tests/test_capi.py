@@ -55,7 +55,7 @@ def _ws(cfg):
     dict(d_model=96, heads=3),            # head_dim 32 not supported in bf16
     dict(layers=0), dict(vocab=1), dict(batch=0),
     dict(d_ff=100),                       # not a multiple of 8
-    dict(d_model=4096, heads=32),         # wider than the LN kernels support
+    dict(d_model=8192, heads=64),         # wider than the LN kernels support
     dict(variant="falplus", reuse_layer=3),   # reuses a block the 2-layer stack does not have
     dict(reuse_layer=2),                  # reuse_layer applies to FAL+ only
     dict(clip_norm=-1.0),
