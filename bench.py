@@ -18,6 +18,9 @@ One JSON line carries, besides the headline (timed with profiling off):
   fal_serial    the same FAL stack with both branches on one stream (isolates
                 the branch concurrency of Sec. 4.2 from the fused residual GEMM);
   gpt_baseline  the same library's sequential GPT stack on the same shape;
+  chunked_head  the headline step with the chunked LM head (head_chunk
+                vocabulary columns per chunk: the logits are never stored
+                whole), its workspace beside the stored-logits one;
   configs       the other benchmark shapes (GPT-2 small / medium / XL): FAL or
                 FAL+ beside GPT, tokens/s and fraction of peak;
   attention_isolated  forward and backward attention kernels timed alone on one
@@ -55,6 +58,7 @@ CONFIG_ARMS = (("gpt2_small", ("fal", "gpt")), ("gpt2_medium", ("falplus", "gpt"
                ("gpt2_xl", ("fal", "falplus", "gpt")))
 REF_SEQ = 128          # tokens per timed step of the reference (oracle) arm
 CPU_SEQ = 512          # tokens of the oracle step timed for cpu_baseline
+HEAD_CHUNK = 8192      # vocabulary columns per chunk of the chunked-LM-head arm
 
 
 def parse(argv=None):
@@ -313,16 +317,23 @@ def init_flat_params(model, s, seed, torch):
 class Arm:
     """One model of the library on the device with its resident inputs."""
 
-    def __init__(self, s, variant, schedule, torch, fal, dev, rank):
+    def __init__(self, s, variant, schedule, torch, fal, dev, rank, head_chunk=0):
         hp = synth.adamw_hparams()
         cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
-                              precision="bf16", schedule=schedule, **hp)
+                              precision="bf16", schedule=schedule, head_chunk=head_chunk, **hp)
+        self.workspace_bytes = fal.workspace_size(cfg)
         self.s, self.variant, self.schedule, self.torch, self.fal, self.dev = s, variant, schedule, torch, fal, dev
         self.m = fal.Model(cfg, device=dev)
         init_flat_params(self.m, s, 1234 + rank, torch)
         self.tok_np, self.tgt_np = synth.make_tokens(s, 1234 + rank)
         self.tok = torch.from_numpy(self.tok_np).to(dev)
         self.tgt = torch.from_numpy(self.tgt_np).to(dev)
+
+    @staticmethod
+    def workspace_of(s, variant, schedule, fal, head_chunk):
+        return fal.workspace_size(fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch,
+                                                  s.vocab, precision="bf16", schedule=schedule,
+                                                  head_chunk=head_chunk, **synth.adamw_hparams()))
 
     def steps(self, k):
         for _ in range(k):
@@ -551,6 +562,14 @@ def main():
         a.close()
         out["gpt_baseline"] = dict(arm_summary(s, r, n, peaks), schedule="serial")
         out["speedup_vs_gpt"] = out["gpt_baseline"]["ms_per_step"] / ms
+        # the same step with the chunked LM head (logits never stored whole)
+        ws_stored = Arm.workspace_of(s, args.variant, args.schedule, fal, 0)
+        a = Arm(s, args.variant, args.schedule, torch, fal, dev, rank, head_chunk=HEAD_CHUNK)
+        r = a.timed(k, w, world)
+        a.close()
+        out["chunked_head"] = dict(arm_summary(s, r, n, peaks), schedule=args.schedule, head_chunk=HEAD_CHUNK,
+                                   workspace_gib=a.workspace_bytes / 2**30, stored_logits_workspace_gib=ws_stored / 2**30,
+                                   vs_stored_logits=ms / r["ms"])
     if not args.no_configs and extra and args.layers is None and args.batch is None:
         cfgs = {}
         for name, variants in CONFIG_ARMS:

@@ -87,6 +87,15 @@ typedef struct fal_config {
     int kv_heads;     /* grouped-query attention (App. E): key/value heads, each shared by
                          heads / kv_heads query heads; 0 = heads (multi-head attention).
                          The fused QKV matrix then has d_model + 2 * kv_heads * head_dim rows. */
+    int head_chunk;   /* 0: the LM head stores the logits [B*T, vocab] once and the cross-entropy
+                         reads them.  > 0 (a multiple of 64): the logits are never stored whole.
+                         The forward's LM-head GEMM reduces each row to its log-sum-exp and
+                         target logit in the epilogue; the backward recomputes the logits
+                         head_chunk vocabulary columns at a time, turns them into the loss
+                         gradient in the epilogue and feeds that chunk to the weight and input
+                         gradients.  The workspace then holds two [B*T, head_chunk] chunks
+                         instead of two [B*T, vocab] arrays, for one more LM-head GEMM per
+                         step.  The "logits" tap is unavailable in this mode. */
 } fal_config;
 
 typedef struct fal_tensor_info {

@@ -394,6 +394,33 @@ __global__ void __launch_bounds__(256) ce_kernel(int rows, int V, long ld, const
   for (int c = V + threadIdx.x; c < ld; c += blockDim.x) dx[c] = from_f<act_t>(0.f);
 }
 
+// Loss of the chunked LM head, one thread per row: the per-slice (max, sum of
+// exp(x - max)) pairs of the logits GEMM's epilogue merge into
+// lse = M + log(sum_j s_j exp(m_j - M)), and loss_row = lse - (target logit).
+// The statistics are slice-major, so a warp reads 32 consecutive rows.
+__global__ void __launch_bounds__(128) ce_combine_kernel(int rows, int nsl, const float2* __restrict__ st, long ld,
+                                                         const float* __restrict__ tl, const int32_t* __restrict__ tgt,
+                                                         int V, float* __restrict__ lse, float* __restrict__ loss_rows,
+                                                         int* err) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= rows) return;
+  float m = -INFINITY, s = 0.f;
+#pragma unroll 4
+  for (int j = 0; j < nsl; ++j) {
+    const float2 v = st[(long)j * ld + r];
+    const float mn = fmaxf(m, v.x);
+    s = s * __expf(m - mn) + v.y * __expf(v.x - mn);
+    m = mn;
+  }
+  const float l = m + logf(s);
+  lse[r] = l;
+  const int t = tgt[r];
+  float x = 0.f;
+  if (t < 0 || t >= V) set_dev_err(err, DEV_ERR_TOKEN);
+  else x = tl[r];
+  loss_rows[r] = l - x;
+}
+
 __global__ void mean_kernel(int n, const float* __restrict__ x, float* __restrict__ out) {
   __shared__ float sh[32];
   float s = 0.f;
@@ -644,6 +671,15 @@ int embed_bwd(int B, int T, int d, int V, const int32_t* tok, const float* dX, f
   if (rows <= 0) return 0;
   embed_bwd_pos_kernel<<<grid_for((long)T * d, 256), 256, 0, s>>>(B, T, d, dX, dwpe);
   embed_bwd_tok_kernel<<<rows, 256, 0, s>>>(rows, d, tok, dX, dwte, V);
+  count_launches(2);
+  return last_err();
+}
+
+int ce_combine(int rows, int nslices, const float2* stats, long ld, const float* tlogit, const int32_t* tgt, int V,
+               float* lse, float* loss_rows, float* loss, int* err, cudaStream_t s) {
+  if (rows <= 0) return 0;
+  ce_combine_kernel<<<(rows + 127) / 128, 128, 0, s>>>(rows, nslices, stats, ld, tlogit, tgt, V, lse, loss_rows, err);
+  mean_kernel<<<1, 1024, 0, s>>>(rows, loss_rows, loss);
   count_launches(2);
   return last_err();
 }

@@ -15,16 +15,19 @@ template <> __device__ __forceinline__ float epi_gelu_grad<bf16>(float x) { retu
 
 // ---- compile-time specialised epilogue arithmetic
 // Which inputs an epilogue reads, as bits of a compile-time KIND.
-// EK_ADAMW (a weight gradient with the optimizer update fused) reads nothing
-// else and is never part of EK_ANY.
+// EK_ADAMW (a weight gradient with the optimizer update fused) and the two
+// cross-entropy epilogues of the LM head read nothing else and are never part
+// of EK_ANY.
 enum EpiKind {
   EK_BIAS = 1, EK_BIAS2 = 2, EK_DGELU = 4, EK_PRE = 8, EK_RESID = 16, EK_RESID2 = 32, EK_GELU = 64,
   EK_ANY = 127,  // every input present-or-null, tested at run time
-  EK_ADAMW = 128
+  EK_ADAMW = 128, EK_CEGRAD = 256, EK_CESTATS = 512
 };
 
 __host__ __device__ inline int epi_kind(const EpiParams& e) {
   if (e.op == EPI_ADAMW) return EK_ADAMW;
+  if (e.op == EPI_CE_GRAD) return EK_CEGRAD;
+  if (e.op == EPI_CE_STATS) return EK_CESTATS;
   return (e.bias ? EK_BIAS : 0) | (e.bias2 ? EK_BIAS2 : 0) | (e.op == EPI_DGELU ? EK_DGELU : 0) |
          (e.pre_f32 ? EK_PRE : 0) | (e.resid ? EK_RESID : 0) | (e.resid2 ? EK_RESID2 : 0) |
          (e.op == EPI_GELU ? EK_GELU : 0);
@@ -148,6 +151,13 @@ __device__ __forceinline__ void epi_math4(const EpiParams& e, int M, int N, int 
   }
 }
 
+// Gradient of the mean cross-entropy for one logit x of row `row`, column c of
+// the chunk: (softmax - one-hot) / rows, with the row's log-sum-exp lse and
+// target column t (vocabulary index minus the chunk's first one).
+__device__ __forceinline__ float ce_grad1(float x, float lse, int t, int c, float scale) {
+  return (__expf(x - lse) - (c == t ? 1.f : 0.f)) * scale;
+}
+
 // Applies the epilogue to NV consecutive accumulator columns [col0, col0+NV)
 // of one output row.  Handles the ragged N edge per element.
 template <typename act_t, int NV>
@@ -155,6 +165,13 @@ __device__ __forceinline__ void epi_row(const EpiParams& e, int M, int N, int ro
                                         float* v) {
   if (row >= M) return;
   const bool full = (col0 + NV <= N);
+  if (e.op == EPI_CE_GRAD) {
+    const float lse = e.ce_lse[row];
+    const int t = e.ce_tgt[row] - e.ce_v0;
+    act_t* o = reinterpret_cast<act_t*>(e.out) + (long)row * e.ldo;
+    for (int j = 0; j < NV && col0 + j < N; ++j) o[col0 + j] = from_f<act_t>(ce_grad1(v[j], lse, t, col0 + j, e.ce_scale));
+    return;
+  }
 #pragma unroll
   for (int j0 = 0; j0 < NV; j0 += 4) {
     const int c = col0 + j0;

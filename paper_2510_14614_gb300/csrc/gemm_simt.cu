@@ -21,6 +21,36 @@ __device__ __forceinline__ float ld_op(const GemmOperand& o, int row, int k, int
   return to_f(o.mn_major ? p[(long)k * o.ld + row] : p[(long)row * o.ld + k]);
 }
 
+// EPI_CE_STATS of one 64 x 64 tile: every row's maximum and sum of exp(x - max)
+// over the tile's columns below N, reduced over the 16 threads that share the
+// row (lanes that differ in tx only), and the logit of the row's target.
+__device__ __forceinline__ void simt_ce_stats(const EpiParams& e, int M, int N, int m0, int n0, int ty, int tx,
+                                              const float (*acc)[4]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = m0 + ty * 4 + i;
+    float m = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (n0 + tx * 4 + j < N) m = fmaxf(m, acc[i][j]);
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (n0 + tx * 4 + j < N) s += __expf(acc[i][j] - m);
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (row < M) {
+      if (tx == 0) e.ce_stats[(long)(n0 / kCeSliceSimt) * e.ce_ld + row] = make_float2(m, s);
+      const int t = e.ce_tgt[row] - e.ce_v0 - n0 - tx * 4;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (t == j && n0 + tx * 4 + j < N) e.ce_tlogit[row] = acc[i][j];
+    }
+  }
+}
+
 template <typename in_t, typename act_t>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const __grid_constant__ SimtParams p) {
   __shared__ float As[SB_K][SB_M + 4];
@@ -56,6 +86,10 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __grid_constant__ 
       }
       __syncthreads();
     }
+  }
+  if (G.epi.op == EPI_CE_STATS) {
+    simt_ce_stats(G.epi, G.M, G.N, m0, n0, ty, tx, acc);
+    return;
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) epi_row<act_t, 4>(G.epi, G.M, G.N, m0 + ty * 4 + i, n0 + tx * 4, acc[i]);

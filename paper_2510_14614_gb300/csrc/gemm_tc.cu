@@ -273,11 +273,29 @@ __device__ __forceinline__ void epi_chunk(const TcParams& p, const EpiParams* ep
   }
   const int row = row0 + lane;
   float4 y[8];
+  if constexpr (KIND == EK_CEGRAD) {
+    // (softmax - one-hot) / rows of this lane's row, zero outside M x N
+    float lse = 0.f;
+    int t = -1;
+    if (row < o.M) { lse = ep->ce_lse[row]; t = ep->ce_tgt[row] - ep->ce_v0; }
+    const float sc = ep->ce_scale;
 #pragma unroll
-  for (int g = 0; g < 8; ++g)
-    y[g] = epi_value4<act_t, KIND>(q, o.M, o.N, row, col0 + 4 * g,
-                                   make_float4(__uint_as_float(r[4 * g]), __uint_as_float(r[4 * g + 1]),
-                                               __uint_as_float(r[4 * g + 2]), __uint_as_float(r[4 * g + 3])));
+    for (int g = 0; g < 8; ++g) {
+      float v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int c = col0 + 4 * g + j;
+        v[j] = (row < o.M && c < o.N) ? ce_grad1(__uint_as_float(r[4 * g + j]), lse, t, c, sc) : 0.f;
+      }
+      y[g] = make_float4(v[0], v[1], v[2], v[3]);
+    }
+  } else {
+#pragma unroll
+    for (int g = 0; g < 8; ++g)
+      y[g] = epi_value4<act_t, KIND>(q, o.M, o.N, row, col0 + 4 * g,
+                                     make_float4(__uint_as_float(r[4 * g]), __uint_as_float(r[4 * g + 1]),
+                                                 __uint_as_float(r[4 * g + 2]), __uint_as_float(r[4 * g + 3])));
+  }
   uint8_t* sb = reinterpret_cast<uint8_t*>(stage);
   const bool gelu = (KIND & EK_GELU) && (KIND != EK_ANY || o.gelu);
   if (o.out_f32) {
@@ -390,6 +408,48 @@ __device__ __forceinline__ void rowdot_store(const EpiParams* ep, int M, int row
   ep->rd_out[((long)(row / T) * ep->rd_H + h) * T + row % T] = s;
 }
 
+// EPI_CE_STATS: folds one 32-column chunk of this lane's row (the columns below
+// N) into the running maximum m and sum s of exp(x - m), and stores the logit of
+// the row's target t (a column of this group) when the chunk holds it.
+__device__ __forceinline__ void ce_stats_chunk(const EpiParams* ep, int M, int N, int row, int col0, int t,
+                                               const uint32_t* r, float& m, float& s) {
+  if (row >= M) return;
+  const int nv = N - col0;  // >= 1: chunks at or beyond N are skipped
+  float cm = m;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (j < nv) cm = fmaxf(cm, __uint_as_float(r[j]));
+  float acc = s * __expf(m - cm);  // 0 on the first chunk (s = 0, m = -inf)
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (j < nv) acc += __expf(__uint_as_float(r[j]) - cm);
+  m = cm;
+  s = acc;
+  const int tc = t - col0;
+  if (tc >= 0 && tc < 32 && tc < nv) {
+    float v = 0.f;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v = (j == tc) ? __uint_as_float(r[j]) : v;
+    ep->ce_tlogit[row] = v;
+  }
+}
+
+// EPI_CE_STATS over one epilogue warp's 32 x 128 piece of a tile (this lane's
+// row `row`, columns col0 .. col0 + 127 at TMEM address taddr): one statistics
+// pair per row for the slice.
+__device__ __noinline__ void ce_stats_tile(const EpiParams* ep, int M, int N, int row, int col0, uint32_t taddr) {
+  const int t = row < M ? ep->ce_tgt[row] - ep->ce_v0 : -1;
+  float m = -INFINITY, s = 0.f;
+  for (int c = 0; c < kCeSliceTc / 32; ++c) {
+    if (col0 + c * 32 >= N) break;
+    uint32_t r[32];
+    TMEM_LD32(taddr + c * 32, r);
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    ce_stats_chunk(ep, M, N, row, col0 + c * 32, t, r, m, s);
+  }
+  if (row < M && col0 < N) ep->ce_stats[(long)(col0 / kCeSliceTc) * ep->ce_ld + row] = make_float2(m, s);
+}
+
 // Runs one chunk with the specialisation the group was prepared for.
 template <typename act_t>
 __device__ __forceinline__ void epi_chunk_dispatch(int kind, const TcParams& p, const EpiParams* ep, const EpiIn q,
@@ -404,6 +464,7 @@ __device__ __forceinline__ void epi_chunk_dispatch(int kind, const TcParams& p, 
     case EK_BIAS | EK_BIAS2 | EK_RESID:
       epi_chunk<act_t, EK_BIAS | EK_BIAS2 | EK_RESID>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
     case EK_ADAMW: epi_chunk<act_t, EK_ADAMW>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
+    case EK_CEGRAD: epi_chunk<act_t, EK_CEGRAD>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
     default: epi_chunk<act_t, EK_ANY>(p, ep, q, o, stage, stage_s, lane, row0, col0, r); break;
   }
 }
@@ -617,6 +678,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       }
       const bool rd = G.epi.rd_out != nullptr;
       float rdot = 0.f;
+      if (kind == EK_CESTATS) ce_stats_tile(&G.epi, eo.M, eo.N, m0 + q * 32 + lane, n0 + half * (TC_BN / 2),
+                                            tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2)));
+      else
       for (int c = 0; c < TC_BN / 64; ++c) {
         const int col0 = n0 + half * (TC_BN / 2) + c * 32;
         if (col0 >= eo.N) break;
@@ -857,6 +921,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(TC_THREADS, 1)
       const int row0 = m0 + (int)rank * 128 + q * 32;
       const bool rd = G.epi.rd_out != nullptr;
       float rdot = 0.f;
+      if (kind == EK_CESTATS) ce_stats_tile(&G.epi, eo.M, eo.N, row0 + lane, n0 + half * (TC_BN / 2),
+                                            tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + half * (TC_BN / 2)));
+      else
       for (int c = 0; c < TC_BN / 64; ++c) {
         const int col0 = n0 + half * (TC_BN / 2) + c * 32;
         if (col0 >= eo.N) break;
@@ -1178,8 +1245,16 @@ int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, st
     {
       const int k = epi_kind(e);
       const bool special = k == 0 || k == EK_BIAS || k == (EK_BIAS | EK_GELU) || k == EK_DGELU ||
-                           k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID) || k == EK_ADAMW;
+                           k == (EK_BIAS | EK_RESID) || k == (EK_BIAS | EK_BIAS2 | EK_RESID) || k == EK_ADAMW ||
+                           k == EK_CEGRAD || k == EK_CESTATS;
       T.kind = special ? k : EK_ANY;
+    }
+    if ((e.op == EPI_CE_GRAD || e.op == EPI_CE_STATS) &&
+        (e.bias || e.bias2 || e.resid || e.resid2 || e.pre_f32 || e.rd_out || e.ord_role || !e.ce_tgt ||
+         (e.op == EPI_CE_GRAD ? (e.out_mode != OUT_ACT || !e.out || !e.ce_lse)
+                              : (e.out != nullptr || !e.ce_stats || !e.ce_tlogit || e.ce_ld < G.M)))) {
+      if (msg) *msg = "cross-entropy epilogue needs its row vectors, a plain output (gradient) or none (statistics)";
+      return 1;
     }
     if (e.rd_out && (e.op != EPI_NONE || e.bias || e.bias2 || e.resid || e.resid2 || e.pre_f32 ||
                      e.out_mode != OUT_ACT || e.rd_hd <= 0 || e.rd_hd % 32 || G.N % e.rd_hd || e.rd_T <= 0 ||

@@ -20,7 +20,9 @@ enum DevErr { DEV_OK = 0, DEV_ERR_TOKEN = 1, DEV_ERR_TIMEOUT = 2 };
 // order).
 // EPI_ADAMW: the GEMM computes the gradient of a weight matrix (stored to `out`,
 // fp32, OUT_F32) and the epilogue also applies AdamW to that weight in place.
-enum EpiOp { EPI_NONE = 0, EPI_GELU = 1, EPI_DGELU = 2, EPI_ADAMW = 3 };
+// EPI_CE_STATS / EPI_CE_GRAD: the LM head's cross-entropy without stored
+// logits (fields ce_* below).
+enum EpiOp { EPI_NONE = 0, EPI_GELU = 1, EPI_DGELU = 2, EPI_ADAMW = 3, EPI_CE_STATS = 4, EPI_CE_GRAD = 5 };
 enum OutMode { OUT_ACT = 0, OUT_F32 = 1, OUT_F32_ACCUM = 2 };
 
 struct EpiParams {
@@ -50,6 +52,15 @@ struct EpiParams {
   // its partial, so the sum is formed in a fixed order.  ord_cap: ints in
   // ord_flags; ord_epoch must differ from every value left by earlier launches.
   int ord_role; int* ord_flags; int ord_cap; int ord_epoch;
+  // Cross-entropy of the LM head (C = logits, column c is vocabulary entry
+  // ce_v0 + c; the target of row r is ce_tgt[r]):
+  // EPI_CE_STATS stores nothing to `out`; for every row and slice of
+  // kCeSliceTc (tcgen05) or kCeSliceSimt (SIMT) columns it writes
+  // ce_stats[slice * ce_ld + r] = (max, sum of exp(x - max)) over the slice's
+  // columns below N (ce_ld >= M), and the logit of the row's target, when it
+  // lies in [ce_v0, ce_v0 + N), to ce_tlogit[r].  EPI_CE_GRAD stores out = (exp(x - ce_lse[r]) - [ce_v0 + c ==
+  // ce_tgt[r]]) * ce_scale (activation type): the gradient of the mean loss.
+  const int* ce_tgt; const float* ce_lse; float2* ce_stats; float* ce_tlogit; long ce_ld; int ce_v0; float ce_scale;
 };
 enum OrdRole { ORD_NONE = 0, ORD_SIGNAL = 1, ORD_WAIT = 2 };
 
@@ -68,6 +79,9 @@ int gemm_tc(const GemmCall& c, int* dev_err, cudaStream_t s, std::string* msg);
 // tiles).
 enum TcKind { TC_ONE = 0, TC_PAIR = 1 };
 int gemm_tc_engine(const GemmCall& c, int kind, int* dev_err, cudaStream_t s, std::string* msg);
+// Columns per EPI_CE_STATS slice: 128 for the tcgen05 engines (one epilogue
+// warp's half of a 256-column tile), 64 for the SIMT GEMM (its tile width).
+constexpr int kCeSliceTc = 128, kCeSliceSimt = 64;
 
 // ---------------------------------------------------------------- attention
 // qkv: activation [B*T, 3*H*hd] (q | k | v, head-major inside each third);
@@ -155,6 +169,11 @@ int embed_bwd(int B, int T, int d, int V, const int32_t* tok, const float* dX, f
 // logits/dlogits: activation [rows, ld] with V valid columns; loss_rows fp32 [rows].
 int cross_entropy(int act_bf16, int rows, int V, long ld, const void* logits, const int32_t* tgt,
                   void* dlogits, float* loss_rows, float* loss, int* err, cudaStream_t s);
+// Loss of the chunked LM head from the EPI_CE_STATS output of the logits GEMM
+// (nslices slices per row, slice-major with row pitch ld): lse and loss_rows
+// fp32 [rows], loss = their mean; a target outside [0, V) sets DEV_ERR_TOKEN.
+int ce_combine(int rows, int nslices, const float2* stats, long ld, const float* tlogit, const int32_t* tgt, int V,
+               float* lse, float* loss_rows, float* loss, int* err, cudaStream_t s);
 // dst += src * colvec (per column), fp32 [rows, d]
 int add_scaled_cols(int rows, int d, const float* src, const float* colvec, float* dst, cudaStream_t s);
 // gscale: device scalar multiplying every gradient (gradient clipping), or null.

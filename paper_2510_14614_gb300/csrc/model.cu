@@ -116,6 +116,12 @@ struct fal_handle {
   void* xf = nullptr;
   float *lnf_mean = nullptr, *lnf_rstd = nullptr;
   void *logits = nullptr, *dlogits = nullptr;
+  // chunked LM head (head_chunk > 0): two [BT, hc] chunk buffers, the
+  // epilogue's per-slice statistics, the target logits and the log-sum-exp
+  int hc = 0, ce_nsl = 0;
+  void* hbuf[2] = {nullptr, nullptr};
+  float2* ce_stats = nullptr;
+  float *ce_tlogit = nullptr, *ce_lse = nullptr;
   float *dX = nullptr, *dY = nullptr, *dA = nullptr, *dU = nullptr, *dU2 = nullptr, *dA1hat = nullptr;
   void *dX_act = nullptr, *dY_act = nullptr, *dA_act = nullptr, *dctx = nullptr, *dh = nullptr, *dqkv = nullptr;
   float *dvec = nullptr, *part0 = nullptr, *part1 = nullptr;
@@ -262,6 +268,10 @@ int validate(const fal_config* c, std::string* msg) {
     *msg = "kv_heads must be 0 (one per head) or divide heads";
     return FAL_ERR_ARG;
   }
+  if (c->head_chunk < 0 || c->head_chunk % 64) {
+    *msg = "head_chunk must be 0 (stored logits) or a positive multiple of 64";
+    return FAL_ERR_ARG;
+  }
   if (c->precision != FAL_BF16 && c->precision != FAL_FP32_DEBUG) { *msg = "bad precision"; return FAL_ERR_ARG; }
   if (c->schedule != FAL_SCHED_SERIAL && c->schedule != FAL_SCHED_TWO_STREAM) { *msg = "bad schedule"; return FAL_ERR_ARG; }
   const int hd = c->d_model / c->heads;
@@ -288,6 +298,8 @@ void init_dims(fal_handle* h, const fal_config* c) {
   h->reuse = c->reuse_layer > 1 ? c->reuse_layer - 1 : 0;
   h->Hkv = c->kv_heads > 0 ? c->kv_heads : h->H;
   h->DQ = h->d + 2 * h->Hkv * h->hd;
+  h->hc = c->head_chunk > 0 ? (c->head_chunk < h->Vp ? c->head_chunk : (int)h->Vp) : 0;
+  h->ce_nsl = (c->vocab + (h->bf ? kCeSliceTc : kCeSliceSimt) - 1) / (h->bf ? kCeSliceTc : kCeSliceSimt);
 }
 
 // MLP-input rule of block i (the block equations of each variant).
@@ -358,8 +370,16 @@ void carve(fal_handle* h, uint8_t* base) {
   h->xf = b.take<uint8_t>(BT * d * a);
   h->lnf_mean = b.take<float>(BT);
   h->lnf_rstd = b.take<float>(BT);
-  h->logits = b.take<uint8_t>((size_t)BT * h->Vp * a);
-  h->dlogits = b.take<uint8_t>((size_t)BT * h->Vp * a);
+  if (h->hc) {
+    h->hbuf[0] = b.take<uint8_t>((size_t)BT * h->hc * a);
+    h->hbuf[1] = b.take<uint8_t>((size_t)BT * h->hc * a);
+    h->ce_stats = b.take<float2>((size_t)h->ce_nsl * BT);
+    h->ce_tlogit = b.take<float>(BT);
+    h->ce_lse = b.take<float>(BT);
+  } else {
+    h->logits = b.take<uint8_t>((size_t)BT * h->Vp * a);
+    h->dlogits = b.take<uint8_t>((size_t)BT * h->Vp * a);
+  }
   h->dX = b.take<float>(BT * d);
   h->dY = b.take<float>(BT * d);
   h->dA = b.take<float>(BT * d);
@@ -712,6 +732,21 @@ int forward_impl(fal_handle* h, const int32_t* tokens, const int32_t* targets) {
   for (int i = 0; i < h->L && c.ok(); ++i) layer_forward(c, i);
   ln_fwd_(c, s, h->Xout, Pp(h, h->lnf_g), Pp(h, h->lnf_b), h->xf, nullptr, h->lnf_mean, h->lnf_rstd, nullptr, nullptr,
           nullptr, nullptr);
+  if (h->hc) {
+    // logits = xf wte^T reduced in the GEMM epilogue to per-slice (max, sum
+    // exp) and the target logit; the loss and lse follow from those
+    EpiParams e = epi_out(nullptr, 0, OUT_ACT);
+    e.op = EPI_CE_STATS;
+    e.ce_tgt = h->tgt; e.ce_stats = h->ce_stats; e.ce_tlogit = h->ce_tlogit; e.ce_ld = h->BT; e.ce_v0 = 0;
+    gemm(c, call1((int)h->BT, h->V, seg(h->xf, h->d, 0, Wp(h, h->wte), h->d, 0, h->d), e), s,
+         "LM head (loss statistics)");
+    ProfScope ps_ce(h, s, 3, 0.0, "cross-entropy");
+    if (c.ok())
+      c.check(ce_combine((int)h->BT, h->ce_nsl, h->ce_stats, h->BT, h->ce_tlogit, h->tgt, h->V, h->ce_lse,
+                         h->loss_rows, h->loss, h->dev_err, s),
+              "cross-entropy");
+    return c.rc;
+  }
   // logits = xf wte^T (tied LM head), padded row pitch Vp
   gemm(c, call1((int)h->BT, h->V, seg(h->xf, h->d, 0, Wp(h, h->wte), h->d, 0, h->d), epi_out(h->logits, h->Vp, OUT_ACT)),
        s, "LM head");
@@ -889,15 +924,47 @@ void layer_backward(Ctx& c, int i) {
           h->part0, Gp(h, p.ln1_g), Gp(h, p.ln1_b), down_biases(h, i - 1));
 }
 
+// Chunked LM head backward.  Chunk j covers vocabulary rows [j hc, j hc + nc)
+// of wte: its logits are recomputed with the loss-gradient epilogue into
+// chunk buffer j % 2, then dwte rows = chunk^T xf (stores) and dxf (+)= chunk
+// wte rows.  The recompute of chunk j + 1 runs in the same launch as the
+// gradients of chunk j, which read the other buffer.
+void head_backward_chunked(Ctx& c, cudaStream_t s) {
+  fal_handle* h = c.h;
+  const int BT = (int)h->BT, d = h->d, V = h->V, C = h->hc;
+  const int n = (V + C - 1) / C;
+  auto width = [&](int j) { return V - j * C < C ? V - j * C : C; };
+  auto recompute = [&](int j) {
+    EpiParams e = epi_out(h->hbuf[j & 1], C, OUT_ACT);
+    e.op = EPI_CE_GRAD;
+    e.ce_lse = h->ce_lse; e.ce_tgt = h->tgt; e.ce_v0 = j * C; e.ce_scale = 1.f / (float)BT;
+    return call1(BT, width(j), seg(h->xf, d, 0, Wp(h, h->wte + (size_t)j * C * d), d, 0, d), e);
+  };
+  auto grads = [&](int j) {
+    const int nc = width(j);
+    return group_calls(
+        {call1(nc, d, seg(h->hbuf[j & 1], C, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte + (size_t)j * C * d), d, OUT_F32)),
+         call1(BT, d, seg(h->hbuf[j & 1], C, 0, Wp(h, h->wte + (size_t)j * C * d), d, 1, nc),
+               epi_out(h->dU, d, j ? OUT_F32_ACCUM : OUT_F32))});
+  };
+  gemm(c, recompute(0), s, "LM head logits gradient (chunk)");
+  for (int j = 0; j < n && c.ok(); ++j)
+    gemm(c, j + 1 < n ? group_calls({grads(j), recompute(j + 1)}) : grads(j), s, "LM head wgrad + dgrad (chunk)");
+}
+
 int backward_impl(fal_handle* h) {
   Ctx c{h};
   cudaStream_t s = h->sm;
   const int BT = (int)h->BT, d = h->d;
   // LM head: dwte = dlogits^T xf and dxf = dlogits wte in one launch (stores;
   // the embedding adds later)
-  gemm(c, group_calls({call1(h->V, d, seg(h->dlogits, h->Vp, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte), d, OUT_F32)),
-                       call1(BT, d, seg(h->dlogits, h->Vp, 0, Wp(h, h->wte), d, 1, h->V), epi_out(h->dU, d, OUT_F32))}),
-       s, "LM head wgrad + dgrad");
+  if (h->hc) {
+    head_backward_chunked(c, s);
+  } else {
+    gemm(c, group_calls({call1(h->V, d, seg(h->dlogits, h->Vp, 1, h->xf, d, 1, BT), epi_out(Gp(h, h->wte), d, OUT_F32)),
+                         call1(BT, d, seg(h->dlogits, h->Vp, 0, Wp(h, h->wte), d, 1, h->V), epi_out(h->dU, d, OUT_F32))}),
+         s, "LM head wgrad + dgrad");
+  }
   ln_bwd_(c, s, h->dU, nullptr, h->Xout, h->lnf_mean, h->lnf_rstd, Pp(h, h->lnf_g), nullptr, h->dX, h->dX_act,
           h->part0, Gp(h, h->lnf_g), Gp(h, h->lnf_b), down_biases(h, h->L - 1));
   if (h->cfg.variant != FAL_GPT) cudaMemsetAsync(h->dA1hat, 0, (size_t)BT * d * 4, s);
@@ -1054,10 +1121,12 @@ int fal_prefill(fal_handle* h, const int32_t* tokens, float* last_logits) {
           nullptr, nullptr);
   // LM head on the last position of every sequence: rows T-1, 2T-1, ... of xf
   // (row pitch T*d), fp32 logits [B, Vp] in the staging buffer when they fit,
-  // else in the logits buffer (B*Vp fp32 values fit there when T >= 2)
+  // else in the logits buffer or the first chunk buffer of the chunked head
   const size_t need = (size_t)h->B * h->Vp;
-  float* out = need <= h->stage_floats ? h->stage : reinterpret_cast<float*>(h->logits);
-  if (out != h->stage && h->bf && h->T < 2) return fail(h, FAL_ERR_UNSUPPORTED, "prefill logits do not fit the workspace");
+  void* alt = h->hc ? h->hbuf[0] : h->logits;
+  const size_t avail = (size_t)h->BT * (h->hc ? (size_t)h->hc : (size_t)h->Vp) * h->asz / 4;
+  float* out = need <= h->stage_floats ? h->stage : need <= avail ? reinterpret_cast<float*>(alt) : nullptr;
+  if (!out) return fail(h, FAL_ERR_UNSUPPORTED, "prefill logits do not fit the workspace");
   const uint8_t* last = reinterpret_cast<const uint8_t*>(h->xf) + (size_t)(h->T - 1) * d * h->asz;
   gemm(c, call1(h->B, h->V, seg(last, (long)h->T * d, 0, Wp(h, h->wte), d, 0, d), epi_out(out, h->Vp, OUT_F32)), s,
        "LM head (last positions)");
@@ -1242,7 +1311,10 @@ int fal_get_tap(fal_handle* h, const char* name, int layer, float* dst, size_t n
   else if (nm == "g") { if (lay) src = h->la[layer].g; cols = F; ld = F; }
   else if (nm == "a1") { src = h->a1; is_act = 0; }
   else if (nm == "xf") { src = h->xf; }
-  else if (nm == "logits") { src = h->logits; cols = h->V; ld = h->Vp; }
+  else if (nm == "logits") {
+    if (h->hc) return fail(h, FAL_ERR_ARG, "the logits are never stored whole with head_chunk > 0");
+    src = h->logits; cols = h->V; ld = h->Vp;
+  }
   if (!src) return fail(h, FAL_ERR_ARG, "unknown tap or layer (or not present for this variant)");
   if (n != (size_t)BT * cols) return fail(h, FAL_ERR_ARG, "tap size mismatch");
   int r = read_dev_err(h);

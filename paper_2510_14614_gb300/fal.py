@@ -26,7 +26,8 @@ class FalConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("variant", "layers", "d_model", "heads", "d_ff", "seq", "batch", "vocab",
                                             "precision", "schedule")] + \
                [(n, ctypes.c_float) for n in ("lr", "beta1", "beta2", "eps", "weight_decay")] + \
-               [("reuse_layer", ctypes.c_int), ("clip_norm", ctypes.c_float), ("kv_heads", ctypes.c_int)]
+               [("reuse_layer", ctypes.c_int), ("clip_norm", ctypes.c_float), ("kv_heads", ctypes.c_int),
+                ("head_chunk", ctypes.c_int)]
 
 
 class FalTensorInfo(ctypes.Structure):
@@ -126,9 +127,10 @@ def _stream_ptr(s):
 
 def make_config(variant, layers, d_model, heads, d_ff, seq, batch, vocab, precision="bf16", schedule="serial",
                 lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=1e-3, reuse_layer=1, clip_norm=0.0,
-                kv_heads=0):
+                kv_heads=0, head_chunk=0):
     return FalConfig(VARIANT[variant], layers, d_model, heads, d_ff, seq, batch, vocab, PRECISION[precision],
-                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay, reuse_layer, clip_norm, kv_heads)
+                     SCHEDULE[schedule], lr, beta1, beta2, eps, weight_decay, reuse_layer, clip_norm, kv_heads,
+                     head_chunk)
 
 
 def workspace_size(cfg: FalConfig) -> int:

@@ -59,6 +59,7 @@ def _ws(cfg):
     dict(variant="falplus", reuse_layer=3),   # reuses a block the 2-layer stack does not have
     dict(reuse_layer=2),                  # reuse_layer applies to FAL+ only
     dict(clip_norm=-1.0),
+    dict(head_chunk=100), dict(head_chunk=-64),   # chunk width must be a positive multiple of 64
     dict(variant="gpt", layers=-1),
 ])
 def test_workspace_size_rejects_bad_configs(libfal, bad):
@@ -80,6 +81,20 @@ def test_workspace_size_accepts_all_shapes(libfal):
     s = synth.SHAPES["gpt_1p3b"]
     _, n = _ws(fal.make_config("fal", s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab))
     assert n < 120 * 2**30
+
+
+def test_chunked_head_shrinks_the_workspace(libfal):
+    """With head_chunk > 0 the workspace holds two [B*T, head_chunk] chunks
+    and the per-slice statistics instead of two [B*T, vocab] logit arrays."""
+    s = synth.SHAPES["gpt_1p3b"]
+    args = ("fal", s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab)
+    _, full = _ws(fal.make_config(*args))
+    rc, chunked = _ws(fal.make_config(*args, head_chunk=8192))
+    assert rc == 0
+    bt, vp = s.batch * s.seq, (s.vocab + 63) // 64 * 64
+    saved = 2 * bt * vp * 2 - (2 * bt * 8192 * 2 + bt * ((s.vocab + 127) // 128) * 8 + 2 * bt * 4)
+    assert abs((full - chunked) - saved) <= 64 * 1024, (full - chunked, saved)
+    assert full - chunked > 2**30
 
 
 def test_null_arguments_are_rejected(libfal):

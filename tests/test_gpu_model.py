@@ -16,19 +16,19 @@ pytestmark = pytest.mark.gpu
 VARIANTS = synth.VARIANTS
 
 
-def _model(variant, s, schedule="serial", **overrides):
+def _model(variant, s, schedule="serial", head_chunk=0, **overrides):
     from paper_2510_14614_gb300 import fal
-    hp = dict(synth.adamw_hparams(), **overrides)
+    hp = dict(synth.adamw_hparams(), head_chunk=head_chunk, **overrides)
     cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
                           precision=s.precision, schedule=schedule, kv_heads=s.kv_heads, **hp)
     return fal.Model(cfg)
 
 
-def _check_parity(variant, s, tol, schedule="serial", seed=0, check_taps=True, reuse=1):
+def _check_parity(variant, s, tol, schedule="serial", seed=0, check_taps=True, reuse=1, head_chunk=0):
     spec = {"reuse": reuse} if reuse != 1 else {}
     params = synth.perturb_params(synth.init_params(variant, s, seed, **spec), seed)
     tok, tgt = synth.make_tokens(s, seed)
-    m = _model(variant, s, schedule, reuse_layer=reuse)
+    m = _model(variant, s, schedule, reuse_layer=reuse, head_chunk=head_chunk)
     m.set_params(params)
     loss = m.forward(tok, tgt)
     cfg = O.Config.from_shape(variant, s, **spec)
@@ -43,7 +43,8 @@ def _check_parity(variant, s, tol, schedule="serial", seed=0, check_taps=True, r
                 errs[f"{name}{i}"] = rel_fro(m.tap(name, i), ref)
         errs["Xout"] = rel_fro(m.tap("X", s.layers), cache["X"][s.layers])
         errs["xf"] = rel_fro(m.tap("xf"), cache["xf"])
-        errs["logits"] = rel_fro(m.tap("logits"), cache["logits"])
+        if not head_chunk:
+            errs["logits"] = rel_fro(m.tap("logits"), cache["logits"])
         if variant in ("fal", "falplus"):
             errs["a1"] = rel_fro(m.tap("a1"), cache["a1"])
     m.backward()
@@ -338,17 +339,20 @@ def test_bounded_wait_expiry_is_reported_and_the_handle_recovers(stall_rows):
     assert np.isfinite(m.train_step(tok, tgt))
 
 
-@pytest.mark.parametrize("variant,shape,schedule", [("fal", "small", "two_stream"), ("gpt", "small", "serial"),
-                                                    ("falplus", "hd128", "serial"), ("fal", "tiny", "serial"),
-                                                    ("parallel", "small", "two_stream")])
-def test_prefill_last_logits_match_oracle(variant, shape, schedule):
+@pytest.mark.parametrize("variant,shape,schedule,chunk", [("fal", "small", "two_stream", 0),
+                                                          ("gpt", "small", "serial", 0),
+                                                          ("falplus", "hd128", "serial", 0),
+                                                          ("fal", "tiny", "serial", 0),
+                                                          ("parallel", "small", "two_stream", 0),
+                                                          ("fal", "small", "two_stream", 256)])
+def test_prefill_last_logits_match_oracle(variant, shape, schedule, chunk):
     """Forward-only prefill (App. E inference): the logits of every sequence's
     last position against the oracle's forward; no backward state after it."""
     from paper_2510_14614_gb300 import fal
     s = {"small": SMALL, "hd128": HD128}.get(shape) or synth.SHAPES["tiny"].replace(layers=3)
     params = synth.perturb_params(synth.init_params(variant, s, 8), 8)
     tok, tgt = synth.make_tokens(s, 8)
-    m = _model(variant, s, schedule)
+    m = _model(variant, s, schedule, head_chunk=chunk)
     m.set_params(params)
     got = m.prefill(tok)
     _, cache = O.forward(params, O.Config.from_shape(variant, s), tok, tgt)
@@ -396,3 +400,68 @@ WIDE = [synth.Shape("wide_2560", 2, 2560, 20, 4 * 2560, 96, 2, 1000, "bf16"),
 def test_parity_wide_models(variant, schedule, s):
     _check_parity(variant, s.replace(precision="fp32"), 1e-4, schedule=schedule)
     _check_parity(variant, s, 2e-2, schedule=schedule)
+
+
+# ---------------------------------------------------------------- chunked LM head
+# head_chunk > 0: the LM head never stores the logits.  The forward reduces
+# them to the log-sum-exp and the target logit in the GEMM epilogue; the
+# backward recomputes them one vocabulary chunk at a time.  Chunks and slices
+# end ragged: vocab 250 in chunks of 64 (fp32 debug, SIMT slices of 64);
+# vocab 1000 in chunks of 256 and of 192 (a chunk narrower than one 256-wide
+# tile), 128-column slices on the tcgen05 path.
+@pytest.mark.parametrize("variant", ["gpt", "fal", "falplus"])
+def test_chunked_head_fp32_debug_parity(variant):
+    _check_parity(variant, synth.SHAPES["tiny"].replace(vocab=250), 1e-4, head_chunk=64)
+
+
+@pytest.mark.parametrize("variant,schedule,chunk", [("fal", "two_stream", 256), ("gpt", "serial", 192),
+                                                    ("falplus", "serial", 1024)])
+def test_chunked_head_bf16_parity(variant, schedule, chunk):
+    _check_parity(variant, SMALL, 1e-2, schedule=schedule, head_chunk=chunk)
+
+
+def test_chunked_head_full_vocab_parity():
+    """The 1.3B width and vocabulary (50257 = six chunks of 8192 and a ragged
+    one of 1105) at depth 1 on one sequence of 2048 tokens."""
+    s = synth.SHAPES["gpt_1p3b"].replace(layers=1, batch=1)
+    _check_parity("fal", s, 1e-2, schedule="two_stream", check_taps=False, head_chunk=8192)
+
+
+def test_chunked_head_train_step_matches_separate_calls():
+    """fal_train_step with the chunked head (AdamW fused into the block
+    weight-gradient GEMMs) leaves the same parameters as forward + backward +
+    step called one by one; its loss agrees with the stored-logits head's to
+    bf16 rounding (fp32 against bf16-rounded logits)."""
+    s = SMALL
+    params = synth.perturb_params(synth.init_params("fal", s, 5), 5)
+    tok, tgt = synth.make_tokens(s, 5)
+    a, b = _model("fal", s, "two_stream", head_chunk=256), _model("fal", s, "two_stream", head_chunk=256)
+    c = _model("fal", s, "two_stream")
+    for m in (a, b, c):
+        m.set_params(params)
+    for _ in range(3):
+        la, lc = a.train_step(tok, tgt), c.train_step(tok, tgt)
+        lb = b.forward(tok, tgt)
+        b.backward()
+        b.step()
+        assert abs(la - lb) <= 1e-6 * abs(lb)
+        assert abs(la - lc) <= 2e-3 * abs(lc), (la, lc)
+    pa, pb = a.params(), b.params()
+    for k in params:
+        np.testing.assert_allclose(pa[k], pb[k], rtol=1e-5, atol=1e-7, err_msg=k)
+
+
+def test_chunked_head_target_out_of_range_is_reported():
+    from paper_2510_14614_gb300 import fal
+    s = SMALL
+    m = _model("fal", s, head_chunk=256)
+    m.set_params(synth.init_params("fal", s, 0))
+    tok, tgt = synth.make_tokens(s, 0)
+    tgt[1, 7] = s.vocab
+    with pytest.raises(fal.FalError) as e:
+        m.forward(tok, tgt)
+    assert e.value.code == fal.FAL_ERR_ARG
+    tgt[1, 7] = 0
+    assert np.isfinite(m.forward(tok, tgt))
+    with pytest.raises(fal.FalError):
+        m.tap("logits")
