@@ -318,6 +318,15 @@ class Arm:
     """One model of the library on the device with its resident inputs."""
 
     def __init__(self, s, variant, schedule, torch, fal, dev, rank, head_chunk=0):
+        # The weights are drawn with torch's device RNG, whose kernels torch
+        # loads lazily on first use.  When that load happened after the model's
+        # ~39 GB workspace had been allocated, every later step of that model ran
+        # about 2 % slower (same kernels and launch shapes; 110 W more power, so
+        # lower clocks); CUDA_MODULE_LOADING=EAGER removed the difference too.
+        # One draw on a tiny tensor before the workspace exists loads them first.
+        warm = torch.Generator(device=dev)
+        warm.manual_seed(0)
+        torch.empty(16, device=dev).normal_(0.0, 1.0, generator=warm)
         hp = synth.adamw_hparams()
         cfg = fal.make_config(variant, s.layers, s.d_model, s.heads, s.d_ff, s.seq, s.batch, s.vocab,
                               precision="bf16", schedule=schedule, head_chunk=head_chunk, **hp)
