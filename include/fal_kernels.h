@@ -40,8 +40,10 @@ int fal_kernel_attention_fwd(int B, int T, int H, int hd, const void* qkv, void*
 
 /* Backward of fal_kernel_attention_fwd: dqkv (bf16 [B*T, 3*H*hd]) from qkv,
  * ctx, lse and dctx (bf16 [B*T, H*hd]).  scratch: fp32 device buffer of at
- * least fal_kernel_attention_bwd_scratch(B, T, H, hd) = B*H*T floats
- * (overwritten: it receives D = rowsum(dO * O) per query and head). */
+ * least fal_kernel_attention_bwd_scratch(B, T, H, hd) floats, 256-byte aligned
+ * (B*H*T rounded up to a multiple of 64, plus 64): overwritten, it receives
+ * D = rowsum(dO * O) per query and head and then the work counter of the
+ * backward kernel, cleared on `stream` before each launch. */
 size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd);
 int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,
                              const void* dctx, void* dqkv, float* scratch, void* stream);
@@ -57,8 +59,8 @@ int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const
  * Scratch comes from one fixed array of FAL_NOALLOC_ATTN_SCRATCH_FLOATS fp32
  * values (16 MiB) compiled into libfal.so: every GPU that loads the library
  * holds it until the process exits.  The call needs
- * B*H*T <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS and returns
- * FAL_ERR_WORKSPACE (launching nothing) above that.  It never calls cudaMalloc,
+ * fal_kernel_attention_bwd_scratch(B, T, H, hd) <= FAL_NOALLOC_ATTN_SCRATCH_FLOATS
+ * (about B*H*T) and returns FAL_ERR_WORKSPACE (launching nothing) above that.  It never calls cudaMalloc,
  * cudaFree or any allocating routine.  Every call made while `stream` is not
  * being captured looks up the array's device address in the current device's
  * context (cudaGetSymbolAddress), so the address stays right after a device

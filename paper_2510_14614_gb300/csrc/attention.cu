@@ -167,7 +167,8 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
           reinterpret_cast<const bf16*>(ctx), reinterpret_cast<const bf16*>(dctx), dvec, rows, T, H, hd);
       count_launches(1);
     }
-    const int r = attn_bwd2_tc(B, T, H, Hkv, hd, qkv, dctx, lse, dvec, dqkv, dev_err, s, msg);
+    int* counter = reinterpret_cast<int*>(dvec + (rows * H + 63) / 64 * 64);
+    const int r = attn_bwd_tc(B, T, H, Hkv, hd, qkv, dctx, lse, dvec, counter, dqkv, dev_err, s, msg);
     if (r) return r;
     (void)d;
   } else {
@@ -187,7 +188,8 @@ int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const v
 
 // ------------------------------------------------------------ allocation-free entry point
 // Scratch for fal_kernel_attention_bwd_noalloc: a fixed file-scope device array
-// that receives the D = rowsum(dO * O) vector, [B, H, T] fp32.  Host code only
+// that receives the D = rowsum(dO * O) vector, [B, H, T] fp32, followed by the
+// backward kernel's work counter.  Host code only
 // ever sees a stand-in for this symbol, so its device address is looked up
 // with cudaGetSymbolAddress while the caller's device is current.
 #include <cuda.h>
@@ -258,14 +260,15 @@ int noalloc_scratch(cudaStream_t s, float** out) {
 extern "C" int fal_kernel_attention_bwd_noalloc(int B, int T, int H, int hd, const void* qkv, const void* ctx,
                                                 const float* lse, const void* dctx, void* dqkv, void* stream) {
   if (B < 0 || T < 0 || H <= 0 || hd <= 0 || !qkv || !ctx || !lse || !dctx || !dqkv) return FAL_ERR_ARG;
-  const size_t need = (size_t)B * H * T;
+  const size_t need = fal::attn_bwd_scratch_floats(B, T, H);
   if (need > kNoAllocFloats) return FAL_ERR_WORKSPACE;
   float* scratch = nullptr;
   const int rc = noalloc_scratch(reinterpret_cast<cudaStream_t>(stream), &scratch);
   if (rc != FAL_OK) return rc;
   std::string msg;
-  // attn_bwd's first kernel writes every D entry before it is read, so nothing
-  // left in the shared array by an earlier call leaks into this one.
+  // attn_bwd's first kernel writes every D entry before it is read, and the
+  // work counter behind D is cleared before the backward kernel starts, so
+  // nothing left in the shared array by an earlier call leaks into this one.
   const int r = fal::attn_bwd(1, B, T, H, hd, qkv, ctx, lse, dctx, dqkv, scratch, nullptr,
                               reinterpret_cast<cudaStream_t>(stream), &msg);
   return r == 0 ? FAL_OK : r == 1 ? FAL_ERR_ARG : r == 6 ? FAL_ERR_UNSUPPORTED : FAL_ERR_CUDA;

@@ -1,40 +1,51 @@
 // Causal multi-head attention backward on tcgen05 (bf16 operands, fp32
-// accumulation in TMEM), in two passes that each keep their accumulators in
-// TMEM for the whole CTA, so that no atomics and no fp32 dQ buffer are needed:
+// accumulation in TMEM) as one persistent launch over two kinds of work item,
+// each keeping its accumulators in TMEM for the whole item, so that no atomics
+// and no fp32 dQ buffer are needed:
 //
-//   pass KV  one CTA per (128-key block, head); streams the 64-query blocks
-//            that can see those keys:
-//              S^T  = K Q^T,  dP^T = V dO^T                    (TMEM, 2 buffers)
-//              P^T  = 2^(S^T*scale*log2e - lse[q]),  dS^T = P^T (dP^T - D[q])
-//              dV  += P^T dO,  dK += dS^T Q                    (TMEM accumulators)
-//   pass Q   one CTA per (128-query block, head); streams the 64-key blocks
-//            up to the diagonal, recomputes S, dP, P and dS row-wise and
-//            accumulates dQ += dS K.
+//   KV item  (batch, key/value head, 128-key block): resident K and V; streams
+//            the 128-query blocks at or after the diagonal of every query head
+//            of the group:
+//              S^T = K Q^T,  dP^T = V dO^T                       (TMEM)
+//              P^T = 2^(S^T*scale*log2e - lse[q]),  dS^T = P^T (dP^T - D[q])
+//              dV += P^T dO  (P^T from TMEM),  dK += dS^T Q  (dS^T from shared memory)
+//   Q item   (batch, query head, 128-query block): resident Q and dO; streams
+//            the 128-key blocks up to the diagonal, recomputes S, dP, P, dS
+//            row-wise and accumulates dQ += dS K (dS from TMEM).
 //
-// The two passes share one body template and run in one launch (alternating
-// CTAs, heaviest blocks of both first).  Roles per CTA (320 threads):
-//   warp 0      producer: the resident 128-row tiles once (K and V, or Q and
-//               dO), then the streamed 64-row tiles through a 4-stage ring; in
-//               pass KV it also stages lse and D of each query block.
-//   warp 1      MMA issuer (one thread), software-pipelined: S / dP of block
-//               j+1 are issued before the accumulating products of block j,
-//               so the tensor pipe works while the elementwise warps handle j.
-//   warps 2..9  elementwise, two warps per TMEM lane quadrant (32 of the 64
-//               columns each): P and dS in bf16 written back into TMEM over
-//               the scores they came from; the accumulating MMAs read them
-//               from there as their A operand (so only B comes from shared
-//               memory, whose bandwidth bounds these small-N products).  At
-//               the end they scale and store dK, dV or dQ in bf16.
+// Every product has N = 128 (or N = head_dim), the shape the tensor pipe runs
+// at its full rate.  Each CTA (one per SM) walks a fixed list of items: items
+// are ranked heaviest first (by the number of streamed blocks, KV before Q at
+// equal count) and dealt to the CTAs in snake order.  Roles per CTA (320
+// threads):
+//   warp 0      producer: the resident tiles of each item once its
+//               predecessor's last S / dP product has read the old ones, then
+//               the streamed tiles through a ring of stages; for KV items also
+//               lse and D of each query block.
+//   warp 1      MMA issuer (one thread).  KV item, per block j:
+//               dV_j, S_{j+1}, dP_{j+1}, dK_j — the scores of block j+1 are
+//               computed while the elementwise warps finish block j.  Q item:
+//               S_{j+1}, dP_{j+1} as soon as the elementwise warps hold S_j and
+//               dP_j in registers, then dQ_j.  The next item's S_0 and dP_0 run
+//               while the elementwise warps store this item's accumulators.
+//   warps 2..9  elementwise, two warps per TMEM lane quadrant (64 of the 128
+//               streamed columns each), then the item's epilogue: dK (scaled)
+//               and dV, or dQ (scaled), in bf16.
+// TMEM (512 columns): S 0..127, dP 128..255, accumulators from 256 (dV | dK,
+// or dQ followed by the Q item's dS in bf16 pairs).
 // D = rowsum(dO * O) is an input: in the model it comes from the epilogue of the
 // GEMM that produces dO, at the kernel-level entry points from a small pre-pass
-// kernel (attention.cu).  Every mbarrier wait
-// is bounded; on expiry the kernel records DEV_ERR_TIMEOUT, lets its MMAs
-// finish, frees TMEM and returns.
+// kernel (attention.cu).  Every mbarrier wait is bounded; on expiry the kernel
+// records DEV_ERR_TIMEOUT, lets its copies and MMAs finish (again bounded),
+// frees TMEM and returns.
+#include <cudaTypedefs.h>
+
 #include <cstring>
+#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
-#include "tc_ptx.cuh"
+#include "attn_ptx.cuh"
 
 namespace fal {
 
@@ -42,86 +53,130 @@ namespace {
 
 using namespace ptx;
 
-constexpr int AB2_THREADS = 320;
-constexpr int AB2_STAGES = 4;
+constexpr int AB_THREADS = 320;
 
-struct AttnBwd2Params {
-  CUtensorMap qkv128, qkv64;  // [B*T, dq] bf16, dq = (H + 2 Hkv) hd, boxes 64 x 128 and 64 x 64, 128-byte swizzle
-  CUtensorMap do128, do64;    // [B*T, d]  bf16, same boxes
+struct AttnBwdParams {
+  CUtensorMap qkv;            // [B*T, dq] bf16, dq = (H + 2 Hkv) hd, box 64 x 128, 128-byte swizzle
+  CUtensorMap dout;           // [B*T, d]  bf16, same box
+  CUtensorMap dqkv_st;        // dqkv as [B][T][dq] bf16, box 64 x 128 x 1: stores clip at the end of each sequence
   const float* lse;           // [B, H, T] log2 units of the scaled scores
   const float* dvec;          // [B, H, T] rowsum(dO * O)
   bf16* dqkv;                 // [B*T, dq]
-  int T, H, Hkv, nblk;        // Hkv key/value heads (each serves H / Hkv query heads); nblk: 128-row blocks
+  int* next_item;             // work counter, zero at launch
+  int B, T, H, Hkv, nblk;     // Hkv key/value heads (each serves H / Hkv query heads); nblk: 128-row blocks
+  int band;                   // key/value heads per band of the item order
   float scale, scale_log2;
   int* err;
 };
 
-template <int HD, bool KV>
-struct Bwd2Smem {
-  static constexpr int KCH = HD / 64;
-  static constexpr int RES = 128 * 64 * 2;             // [128 rows][64] bf16 chunk (resident tiles)
-  static constexpr int STR = 64 * 64 * 2;              // [64 rows][64] bf16 chunk (streamed tiles)
-  static constexpr int RES_A = 0;                      // K (KV) or Q (Q)
-  static constexpr int RES_B = RES_A + KCH * RES;      // V (KV) or dO (Q)
-  static constexpr int STAGE = 2 * KCH * STR;          // Q | dO (KV) or K | V (Q)
-  static constexpr int ST_OFF = RES_B + KCH * RES;
-  static constexpr int VEC_OFF = ST_OFF + AB2_STAGES * STAGE;  // KV: lse[64] | D[64] per stage
-  static constexpr int BAR_OFF = VEC_OFF + (KV ? AB2_STAGES * 512 : 0);
-  static constexpr int TOTAL = BAR_OFF + 256 + 1024;   // barriers + alignment slack
+template <int HD>
+struct BwdSmem {
+  static constexpr int KCH = HD / 64;                  // 64-column chunks of a head
+  static constexpr int CH = 128 * 64 * 2;              // one [128 rows][64] bf16 chunk, 16 KB
+  static constexpr int STAGES = HD == 64 ? 4 : 2;
+  static constexpr int RES_A = 0;                      // K (KV item) or Q (Q item)
+  static constexpr int RES_B = KCH * CH;               // V or dO
+  static constexpr int HALF = KCH * CH;                // half of a stage: Q | dO (KV) or K | V (Q)
+  static constexpr int ST_OFF = 2 * KCH * CH;
+  static constexpr int STAGE = 2 * HALF;
+  static constexpr int STG_OFF = ST_OFF + STAGES * STAGE;  // epilogue staging: one accumulator in bf16
+  static constexpr int VEC_OFF = STG_OFF + KCH * CH;   // lse[128] | D[128] per stage (KV items)
+  static constexpr int BAR_OFF = VEC_OFF + STAGES * 1024;
+  static constexpr int TOTAL = BAR_OFF + 256;
+  static constexpr int LAUNCH = TOTAL + 1024 < 232448 ? TOTAL + 1024 : 232448;  // + alignment slack
 };
 
-template <int HD, bool KV>
-__device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) {
-  using L = Bwd2Smem<HD, KV>;
-  constexpr int KCH = L::KCH;
+// Item of rank k.  Items come in bands of p.band key/value heads (with their
+// query heads), so that the CTAs working at any time share a few heads' Q, K,
+// V and dO in L2; within a band heaviest first: per level (streamed blocks per
+// query head, nblk down to 1) the band's KV items, then its Q items.
+struct BwdItem {
+  int kv, b, head, blk, nit, nit_h;  // head: key/value head (KV) or query head (Q); blk: 128-row block
+};
+__device__ __forceinline__ BwdItem decode_item(const AttnBwdParams& p, int k) {
+  BwdItem it;
+  const int gs = p.H / p.Hkv;
+  const int per_band = p.nblk * p.band * (1 + gs);
+  const int band = k / per_band, rb = k - band * per_band;
+  const int nb = min(p.band, p.B * p.Hkv - band * p.band);  // key/value heads in this band
+  const int per_level = nb * (1 + gs);
+  const int level = rb / per_level, w = rb - level * per_level;
+  if (w < nb) {
+    const int kvh = band * p.band + w;     // batch-major key/value head index
+    it.kv = 1;
+    it.b = kvh / p.Hkv;
+    it.head = kvh - it.b * p.Hkv;
+    it.blk = level;                        // key block: query blocks blk .. nblk-1 see it
+    it.nit_h = p.nblk - level;
+    it.nit = gs * it.nit_h;
+  } else {
+    const int q = w - nb;
+    const int kvh = band * p.band + q / gs;
+    it.kv = 0;
+    it.b = kvh / p.Hkv;
+    it.head = (kvh - it.b * p.Hkv) * gs + q % gs;
+    it.blk = p.nblk - 1 - level;           // query block: key blocks 0 .. blk
+    it.nit_h = it.nit = it.blk + 1;
+  }
+  return it;
+}
+
+// Unbounded-by-abort wait used while draining after an error: returns when the
+// phase completed or after kWaitNs.
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity) && global_timer_ns() - t0 < kWaitNs) {}
+}
+
+template <int HD>
+__global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_constant__ AttnBwdParams p) {
+  using L = BwdSmem<HD>;
+  constexpr int KCH = L::KCH, NS = L::STAGES, NR = 4;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
+  // the layout needs its start 1024-byte aligned inside the launched size
+  if (base - raw + L::TOTAL > L::LAUNCH) {
+    if (threadIdx.x == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+    return;
+  }
   uint8_t* sbase = smem_raw + (base - raw);
   const uint32_t bar = base + L::BAR_OFF;
-  const uint32_t res_full = bar;
-  auto st_full = [&](int s) { return bar + 8u * (1 + s); };
-  auto st_empty = [&](int s) { return bar + 8u * (1 + AB2_STAGES + s); };
-  auto sdp_full = [&](int b) { return bar + 8u * (1 + 2 * AB2_STAGES + b); };
-  auto ps_full = [&](int b) { return bar + 8u * (3 + 2 * AB2_STAGES + b); };
-  const uint32_t fin = bar + 8u * (5 + 2 * AB2_STAGES), drain = bar + 8u * (6 + 2 * AB2_STAGES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sbase + L::BAR_OFF + 8 * (7 + 2 * AB2_STAGES));
-  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(sbase + L::BAR_OFF + 8 * (7 + 2 * AB2_STAGES) + 4);
+  const uint32_t res_full = bar, res_empty = bar + 8;
+  auto st_full = [&](int s) { return bar + 8u * (2 + s); };
+  auto st_empty = [&](int s) { return bar + 8u * (2 + NS + s); };
+  const uint32_t s_full = bar + 8u * (2 + 2 * NS), dp_full = s_full + 8, rd = s_full + 16, p_full = s_full + 24,
+                 ds_full = s_full + 32, ds_empty = s_full + 40, stg_full = s_full + 48, stg_empty = s_full + 56,
+                 acc_full = s_full + 64, acc_empty = s_full + 72, drain = s_full + 80;
+  auto it_full = [&](int i) { return s_full + 88 + 8u * i; };
+  auto it_empty = [&](int i) { return s_full + 88 + 8u * (NR + i); };
+  uint8_t* misc = sbase + L::BAR_OFF + 8 * (13 + 2 * NS + 2 * NR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc);
+  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(misc + 4);
+  volatile int* ring = reinterpret_cast<volatile int*>(misc + 8);  // item ranks handed from the producer to the other roles
   const float* vec_base = reinterpret_cast<const float*>(sbase + L::VEC_OFF);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  // heaviest CTAs first: key block 0 (pass KV) / the last query block (pass Q)
-  const int blk = KV ? bx : p.nblk - 1 - bx;
-  const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
-  // Grouped-query attention: query head h uses key / value head g.  Pass KV
-  // runs one CTA per key / value head (on the grid row of the group's first
-  // query head) and streams the query blocks of every head of the group, so
-  // dK and dV sum over the group in TMEM.
-  const int gs = p.H / p.Hkv, g = h / gs;
-  if (KV && h % gs) return;
+  const int gs = p.H / p.Hkv;
   const int d = p.H * HD;
-  const long dq = (long)(p.H + 2 * p.Hkv) * HD;    // qkv / dqkv row width
-  const int kcol = d + g * HD, vcol = d + (p.Hkv + g) * HD;
-  const int row_base = b * p.T;
-  const int r0 = blk * 128;  // first key (KV) or query (Q) row of this CTA
-  const int nstream = (p.T + 63) / 64;
-  int j0, nit, nit_h;
-  if (KV) {
-    j0 = r0 / 64;             // query blocks that reach key r0 or later
-    nit_h = nstream - j0;     // per query head of the group
-    nit = gs * nit_h;
-  } else {
-    j0 = 0;                   // key blocks up to the diagonal
-    const int last = min(nstream - 1, (r0 + 127) / 64);
-    nit = nit_h = last + 1;
-  }
+  const int total = p.nblk * p.B * (p.Hkv + p.H);
 
   if (threadIdx.x == 0) {
     mbar_init(res_full, 1);
-    for (int s = 0; s < AB2_STAGES; ++s) { mbar_init(st_full(s), KV ? 2 : 1); mbar_init(st_empty(s), 1); }
-    for (int i = 0; i < 2; ++i) { mbar_init(sdp_full(i), 1); mbar_init(ps_full(i), 8); }
-    mbar_init(fin, 1);
+    mbar_init(res_empty, 1);
+    for (int s = 0; s < NS; ++s) { mbar_init(st_full(s), 2); mbar_init(st_empty(s), 1); }
+    mbar_init(s_full, 1);
+    mbar_init(dp_full, 1);
+    mbar_init(rd, 8);
+    mbar_init(p_full, 8);
+    mbar_init(ds_full, 8);
+    mbar_init(ds_empty, 1);
+    mbar_init(stg_full, 8);
+    mbar_init(stg_empty, 1);
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 8);
     mbar_init(drain, 1);
+    for (int i = 0; i < NR; ++i) { mbar_init(it_full(i), 1); mbar_init(it_empty(i), 9); }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -131,124 +186,209 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // TMEM columns: S buffers 0 / 64, dP buffers 128 / 192, accumulators from 256.
-  // P (KV only) and dS overwrite the first 16 of each warp's 32 score columns
-  // in bf16 pairs: query / key k of a 64 block sits in column 32*(k/32) + (k%32)/2.
-  constexpr uint32_t T_S = 0, T_DP = 128, T_A1 = 256, T_A2 = 256 + HD;
+  // TMEM columns.  KV item: S^T (then P^T in bf16 pairs) 0..127, dP^T (then
+  // dS^T in bf16 pairs) 128..255, dV, dK.  Q item: S, dP, dQ, dS in bf16 pairs.
+  constexpr uint32_t T_S = 0, T_DP = 128, T_A1 = 256, T_A2 = 256 + HD, T_DS = 256 + HD;
+
+  // n-th item of this CTA as handed out by the producer (-1: no more work)
+  auto next_item = [&](int n, bool& ok) -> int {
+    const int i = n % NR;
+    if (!mbar_wait(it_full(i), (n / NR) & 1, abort_flag)) { ok = false; return -1; }
+    return ring[i];
+  };
 
   if (warp == 0) {
     // ------------------------------------------------ producer
     bool ok = true;
-    if (lane == 0) {
-      mbar_arrive_expect_tx(res_full, 2 * KCH * L::RES);
-      for (int c = 0; c < KCH; ++c) {
-        if (KV) {
-          tma_load_2d(base + L::RES_A + c * L::RES, &p.qkv128, kcol + 64 * c, row_base + r0, res_full);
-          tma_load_2d(base + L::RES_B + c * L::RES, &p.qkv128, vcol + 64 * c, row_base + r0, res_full);
-        } else {
-          tma_load_2d(base + L::RES_A + c * L::RES, &p.qkv128, h * HD + 64 * c, row_base + r0, res_full);
-          tma_load_2d(base + L::RES_B + c * L::RES, &p.do128, h * HD + 64 * c, row_base + r0, res_full);
-        }
-      }
-    }
-    // (jj, hq): streamed block index within its query head, and that head
-    // (pass KV walks the heads of the group one after another)
-    for (int it = 0, jj = 0, hq = KV ? g * gs : h; it < nit && ok; ++it) {
-      const int s = it % AB2_STAGES;
-      if (!mbar_wait(st_empty(s), ((it / AB2_STAGES) & 1) ^ 1u, abort_flag)) { ok = false; break; }
-      const int c0 = (j0 + jj) * 64;                   // first streamed row of this block
-      const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
+    int g = 0, n = 0;  // streamed blocks and resident sets issued so far
+    for (int r = 0; ok; ++r) {
+      // take the next item from the launch-wide counter and hand it to the other roles
+      if (!mbar_wait(it_empty(r % NR), ((r / NR) & 1) ^ 1u, abort_flag)) { ok = false; break; }
+      int k = 0;
       if (lane == 0) {
-        mbar_arrive_expect_tx(st_full(s), L::STAGE);
+        k = atomicAdd(p.next_item, 1);
+        if (k >= total) k = -1;
+        ring[r % NR] = k;
+        mbar_arrive(it_full(r % NR));
+      }
+      k = __shfl_sync(0xffffffffu, k, 0);
+      if (k < 0) break;
+      const BwdItem it = decode_item(p, k);
+      const int row_base = it.b * p.T;
+      const int kcol = d + (it.kv ? it.head : it.head / gs) * HD;
+      const int vcol = kcol + p.Hkv * HD;
+      // resident tiles, once the previous item's last S / dP products have read the old ones
+      if (!mbar_wait(res_empty, (n & 1) ^ 1u, abort_flag)) { ok = false; break; }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(res_full, 2 * KCH * L::CH);
         for (int c = 0; c < KCH; ++c) {
-          if (KV) {
-            tma_load_2d(sb + c * L::STR, &p.qkv64, hq * HD + 64 * c, row_base + c0, st_full(s));
-            tma_load_2d(sb + (KCH + c) * L::STR, &p.do64, hq * HD + 64 * c, row_base + c0, st_full(s));
+          if (it.kv) {
+            tma_load_2d(base + L::RES_A + c * L::CH, &p.qkv, kcol + 64 * c, row_base + it.blk * 128, res_full);
+            tma_load_2d(base + L::RES_B + c * L::CH, &p.qkv, vcol + 64 * c, row_base + it.blk * 128, res_full);
           } else {
-            tma_load_2d(sb + c * L::STR, &p.qkv64, kcol + 64 * c, row_base + c0, st_full(s));
-            tma_load_2d(sb + (KCH + c) * L::STR, &p.qkv64, vcol + 64 * c, row_base + c0, st_full(s));
+            tma_load_2d(base + L::RES_A + c * L::CH, &p.qkv, it.head * HD + 64 * c, row_base + it.blk * 128, res_full);
+            tma_load_2d(base + L::RES_B + c * L::CH, &p.dout, it.head * HD + 64 * c, row_base + it.blk * 128, res_full);
           }
         }
       }
-      if (KV) {
-        // lse and D of the block's 64 queries (zero beyond the sequence)
-        float* v = reinterpret_cast<float*>(sbase + L::VEC_OFF + s * 512);
-        for (int i = lane; i < 64; i += 32) {
-          const int t = c0 + i;
-          const long bq = (long)b * p.H + hq;
-          v[i] = t < p.T ? p.lse[bq * p.T + t] : 0.f;
-          v[64 + i] = t < p.T ? p.dvec[bq * p.T + t] : 0.f;
+      __syncwarp();
+      ++n;
+      for (int j = 0, jj = 0, hq = it.kv ? it.head * gs : it.head; j < it.nit; ++j, ++g) {
+        const int s = g % NS;
+        if (!mbar_wait(st_empty(s), ((g / NS) & 1) ^ 1u, abort_flag)) { ok = false; break; }
+        const int c0 = (it.kv ? it.blk + jj : jj) * 128;   // first streamed row of the block
+        const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(st_full(s), L::STAGE);
+          for (int c = 0; c < KCH; ++c) {
+            if (it.kv) {
+              tma_load_2d(sb + c * L::CH, &p.qkv, hq * HD + 64 * c, row_base + c0, st_full(s));
+              tma_load_2d(sb + L::HALF + c * L::CH, &p.dout, hq * HD + 64 * c, row_base + c0, st_full(s));
+            } else {
+              tma_load_2d(sb + c * L::CH, &p.qkv, kcol + 64 * c, row_base + c0, st_full(s));
+              tma_load_2d(sb + L::HALF + c * L::CH, &p.qkv, vcol + 64 * c, row_base + c0, st_full(s));
+            }
+          }
+        }
+        if (it.kv) {
+          // lse and D of the block's 128 queries (zero beyond the sequence): all
+          // eight loads of a lane are in flight together
+          float* v = reinterpret_cast<float*>(sbase + L::VEC_OFF + s * 1024);
+          const float* lsrc = p.lse + ((long)it.b * p.H + hq) * p.T;
+          const float* dsrc = p.dvec + ((long)it.b * p.H + hq) * p.T;
+          float lv[4], dvv[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int t = c0 + lane + 32 * q;
+            lv[q] = t < p.T ? __ldg(lsrc + t) : 0.f;
+            dvv[q] = t < p.T ? __ldg(dsrc + t) : 0.f;
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            v[lane + 32 * q] = lv[q];
+            v[128 + lane + 32 * q] = dvv[q];
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(st_full(s));
+        __syncwarp();
+        if (++jj == it.nit_h) { jj = 0; ++hq; }
       }
-      __syncwarp();
-      if (++jj == nit_h) { jj = 0; ++hq; }
     }
-    if (!ok && lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+    if (!ok) {
+      if (lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
+      // let the copies already issued land before the CTA's shared memory goes away
+      if (n > 0) drain_wait(res_full, (uint32_t)((n - 1) & 1));
+      for (int s = 0; s < NS && s < g; ++s) {
+        const int last = g - 1 - ((g - 1 - s) % NS);      // last block that used stage s
+        drain_wait(st_full(s), (uint32_t)((last / NS) & 1));
+      }
+    }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     bool ok = true, issued = false;
     if (lane == 0) {
-      const uint32_t id_s = make_idesc_bf16(0, 0, 128, 64);    // S, dP: both K-major, N = 64
-      const uint32_t id_acc = make_idesc_bf16(0, 1, 128, HD);  // accumulate: A K-major, B MN-major
-      ok = mbar_wait(res_full, 0, abort_flag);
-      for (int it = 0; it <= nit && ok; ++it) {
-        if (it < nit) {
-          const int bb = it & 1, s = it % AB2_STAGES;
-          // (buffer bb was last read by the accumulating MMAs of block it-2, issued
-          //  earlier by this thread: the tensor pipe runs them in order)
-          if (!mbar_wait(st_full(s), (it / AB2_STAGES) & 1, abort_flag)) { ok = false; break; }
-          tc_fence_after();
+      const uint32_t id_s = make_idesc_bf16(0, 0, 128, 128);   // S, dP: both K-major, N = 128
+      const uint32_t id_acc = make_idesc_bf16(0, 1, 128, HD);  // accumulate: B MN-major
+      // descriptor words: one high word for every operand (stride 1024 between
+      // 8-row groups, 128-byte swizzle); low words step by immediates along K
+      const uint32_t hi = desc_hi(1024);
+      const uint32_t lo_ra = desc_lo(base + L::RES_A, 16), lo_rb = desc_lo(base + L::RES_B, 16);
+      int g = 0, gk = 0, n = 0;
+      // S (from resident A and stage half 0) or dP (resident B, stage half 1) of the block in stage s
+      auto issue_sdp = [&](uint32_t dst, uint32_t lo_res, int s, int half) {
+        const uint32_t lo_st = desc_lo(base + L::ST_OFF + s * L::STAGE + half * L::HALF, 16);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t o = (kk >> 2) * (L::CH >> 4) + (kk & 3) * 2;
+          tc_mma_w(tmem + dst, lo_res + o, lo_st + o, hi, id_s, kk > 0);
+        }
+      };
+      // accumulate A (bf16 pairs in TMEM from column a_col: k at 64*(k/64) + (k%64)/2,
+      // or 32*(k/64) + (k%64)/2 when a_step is 32) times the stage half as MN-major B
+      auto issue_acc = [&](uint32_t dst, uint32_t a_col, uint32_t a_step, uint32_t lo_b, bool acc) {
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          tc_mma_ts_w(tmem + dst, tmem + a_col + a_step * (kk >> 2) + 8 * (kk & 3), lo_b + kk * 128, hi, id_acc,
+                      (acc || kk > 0));
+      };
+      for (int r = 0; ok; ++r) {
+        const int k = next_item(r, ok);
+        if (ok) mbar_arrive(it_empty(r % NR));
+        if (k < 0) break;
+        const BwdItem it = decode_item(p, k);
+        if (!mbar_wait(res_full, n & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(st_full(g % NS), (g / NS) & 1, abort_flag)) { ok = false; break; }
+        if (g > 0 && !mbar_wait(rd, (g - 1) & 1, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        issue_sdp(T_S, lo_ra, g % NS, 0);
+        tc_commit(s_full);
+        issue_sdp(T_DP, lo_rb, g % NS, 1);
+        tc_commit(dp_full);
+        issued = true;
+        if (it.nit == 1) tc_commit(res_empty);
+        for (int j = 0; j < it.nit; ++j, ++g) {
+          const int s = g % NS;
           const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
-#pragma unroll
-          for (int kk = 0; kk < HD / 16; ++kk) {
-            const uint32_t oa = (kk >> 2) * L::RES + (kk & 3) * 32, ob = (kk >> 2) * L::STR + (kk & 3) * 32;
-            tc_mma(tmem + T_S + 64 * bb, smem_desc(base + L::RES_A + oa, 16, 1024), smem_desc(sb + ob, 16, 1024),
-                   id_s, kk > 0);
-          }
-#pragma unroll
-          for (int kk = 0; kk < HD / 16; ++kk) {
-            const uint32_t oa = (kk >> 2) * L::RES + (kk & 3) * 32, ob = (kk >> 2) * L::STR + (kk & 3) * 32;
-            tc_mma(tmem + T_DP + 64 * bb, smem_desc(base + L::RES_B + oa, 16, 1024),
-                   smem_desc(sb + KCH * L::STR + ob, 16, 1024), id_s, kk > 0);
-          }
-          tc_commit(sdp_full(bb));
-          issued = true;
-        }
-        if (it >= 1) {
-          const int jt = it - 1, bj = jt & 1, sj = jt % AB2_STAGES;
-          if (!mbar_wait(ps_full(bj), (jt >> 1) & 1, abort_flag)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t sb = base + L::ST_OFF + sj * L::STAGE;
-#pragma unroll
-          for (int kk = 0; kk < 64 / 16; ++kk) {
-            const uint32_t acol = 64 * bj + (kk >> 1) * 32 + (kk & 1) * 8;  // 16 k values in 8 columns
-            if (KV) {
-              // dV += P^T dO, dK += dS^T Q   (B: the streamed [64 q][hd] tiles read MN-major)
-              tc_mma_ts(tmem + T_A1, tmem + T_S + acol, smem_desc(sb + KCH * L::STR + kk * 2048, L::STR, 1024), id_acc,
-                        (jt > 0 || kk > 0));
-              tc_mma_ts(tmem + T_A2, tmem + T_DP + acol, smem_desc(sb + kk * 2048, L::STR, 1024), id_acc,
-                        (jt > 0 || kk > 0));
-            } else {
-              // dQ += dS K   (B: the streamed [64 keys][hd] tile read MN-major)
-              tc_mma_ts(tmem + T_A1, tmem + T_DP + acol, smem_desc(sb + kk * 2048, L::STR, 1024), id_acc,
-                        (jt > 0 || kk > 0));
+          const uint32_t lo_h0 = desc_lo(sb, L::CH), lo_h1 = desc_lo(sb + L::HALF, L::CH);  // MN-major B
+          const bool more = j + 1 < it.nit;
+          if (it.kv) {
+            // dV += P^T dO
+            if (!mbar_wait(p_full, gk & 1, abort_flag)) { ok = false; break; }
+            if (j == 0 && n > 0 && !mbar_wait(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
+            tc_fence_after();
+            issue_acc(T_A1, T_S, 64, lo_h1, j > 0);
+            if (more) {
+              // S_{j+1} overwrites P^T_j, which the products above read first (in-order pipe)
+              if (!mbar_wait(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
+              tc_fence_after();
+              issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
+              tc_commit(s_full);
             }
+            // dK += dS^T Q   (dS^T in bf16 pairs over the dP^T columns)
+            if (!mbar_wait(ds_full, g & 1, abort_flag)) { ok = false; break; }
+            tc_fence_after();
+            issue_acc(T_A2, T_DP, 64, lo_h0, j > 0);
+            tc_commit(ds_empty);
+            tc_commit(st_empty(s));
+            if (more) {
+              // dP_{j+1} overwrites dS^T_j after the product above has read it
+              issue_sdp(T_DP, lo_rb, (g + 1) % NS, 1);
+              tc_commit(dp_full);
+              if (j + 2 == it.nit) tc_commit(res_empty);
+            }
+            ++gk;
+          } else {
+            if (more) {
+              if (!mbar_wait(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait(rd, g & 1, abort_flag)) { ok = false; break; }
+              tc_fence_after();
+              issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
+              tc_commit(s_full);
+              issue_sdp(T_DP, lo_rb, (g + 1) % NS, 1);
+              tc_commit(dp_full);
+              if (j + 2 == it.nit) tc_commit(res_empty);
+            }
+            // dQ += dS K   (dS in bf16 pairs from column T_DS)
+            if (!mbar_wait(ds_full, g & 1, abort_flag)) { ok = false; break; }
+            if (j == 0 && n > 0 && !mbar_wait(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
+            tc_fence_after();
+            issue_acc(T_A1, T_DS, 32, lo_h0, j > 0);
+            tc_commit(ds_empty);
+            tc_commit(st_empty(s));
           }
-          tc_commit(st_empty(sj));
         }
+        if (!ok) break;
+        tc_commit(acc_full);
+        ++n;
       }
-      if (ok) {
-        tc_commit(fin);
-      } else {
+      if (!ok) {
         set_dev_err(p.err, DEV_ERR_TIMEOUT);
+        *abort_flag = 1;
         if (issued) {
           tc_commit(drain);
-          const uint64_t t0 = global_timer_ns();
-          while (!mbar_try_wait(drain, 0) && global_timer_ns() - t0 < kWaitNs) {}
+          drain_wait(drain, 0);
         }
-        *abort_flag = 1;
       }
     }
     __syncwarp();
@@ -256,102 +396,192 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
     // ------------------------------------------------ elementwise (two warps per lane quadrant)
     const int q4 = warp & 3, half = (warp - 2) >> 2;
     const int r = q4 * 32 + lane;  // TMEM lane = row inside the 128-row block
-    const int row = r0 + r;        // key (KV) or query (Q) position
     const uint32_t lane_addr = tmem + ((uint32_t)(q4 * 32) << 16);
-    float lse_r = 0.f, d_r = 0.f;
-    if (!KV && row < p.T) {
-      lse_r = p.lse[(long)bh * p.T + row];
-      d_r = p.dvec[(long)bh * p.T + row];
-    }
+    const float sl2 = p.scale_log2;
+    const bool storer = warp == 2 && lane == 0;  // issues the epilogue's TMA stores
     bool ok = true;
-    for (int it = 0, jj = -1; it < nit; ++it) {
-      if (++jj == nit_h) jj = 0;  // streamed block index within its query head
-      const int bb = it & 1, s = it % AB2_STAGES;
-      const int c0 = (j0 + jj) * 64 + 32 * half;  // first streamed position of this warp's 32 columns
-      // sdp_full(it) also covers the accumulating MMAs of block it-2, the last
-      // readers of the P / dS columns of buffer bb
-      if (!mbar_wait(sdp_full(bb), (it >> 1) & 1, abort_flag)) { ok = false; break; }
-      if (KV && !mbar_wait(st_full(s), (it / AB2_STAGES) & 1, abort_flag)) { ok = false; break; }
-      tc_fence_after();
-      uint32_t sr[32], dr[32];
-      TMEM_LD32(lane_addr + T_S + 64 * bb + 32 * half, sr);
-      TMEM_LD32(lane_addr + T_DP + 64 * bb + 32 * half, dr);
-      tmem_wait_ld();
-      const float* vl = vec_base + s * 128 + 32 * half;  // KV: lse / D of this warp's 32 queries
-      float pv[32], dv[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int c = c0 + i;
-        float lse, dd;
-        bool masked;
-        if (KV) {
-          lse = vl[i];
-          dd = vl[64 + i];
-          masked = c >= p.T || row >= p.T || c < row;   // query c, key row
-        } else {
-          lse = lse_r;
-          dd = d_r;
-          masked = c >= p.T || row >= p.T || c > row;   // key c, query row
-        }
-        const float pr = masked ? 0.f : ex2_approx(__uint_as_float(sr[i]) * p.scale_log2 - lse);
-        pv[i] = pr;
-        dv[i] = pr * (__uint_as_float(dr[i]) - dd);
-      }
-      // bf16 pairs back into this warp's own score columns (A operands of the accumulating MMAs)
-      uint32_t pw[16], dw[16];
-#pragma unroll
-      for (int w = 0; w < 16; ++w) {
-        __nv_bfloat162 a = __floats2bfloat162_rn(pv[2 * w], pv[2 * w + 1]);
-        __nv_bfloat162 g = __floats2bfloat162_rn(dv[2 * w], dv[2 * w + 1]);
-        pw[w] = *reinterpret_cast<uint32_t*>(&a);
-        dw[w] = *reinterpret_cast<uint32_t*>(&g);
-      }
-      if (KV) TMEM_ST16(lane_addr + T_S + 64 * bb + 32 * half, pw);
-      TMEM_ST16(lane_addr + T_DP + 64 * bb + 32 * half, dw);
-      tmem_wait_st();
-      tc_fence_before();
+    int g = 0, gk = 0, n = 0, su = 0;  // su: uses of the epilogue staging buffer
+    // this thread's part of a row of the staging tile (128-byte swizzle): head_dim
+    // 128: all of chunk `half`; head_dim 64: half of the one chunk
+    uint8_t* stg_row = sbase + L::STG_OFF + (HD == 128 ? half * L::CH : 0) + (r >> 3) * 1024 + (r & 7) * 128;
+    const int u0 = HD == 128 ? 0 : 4 * half;
+    for (int rk = 0; ok; ++rk) {
+      const int k = next_item(rk, ok);
       __syncwarp();
-      if (lane == 0) mbar_arrive(ps_full(bb));
-    }
-    // ------------------------------------------------ results: dK (scaled) and dV, or dQ (scaled)
-    if (ok && mbar_wait(fin, 0, abort_flag)) {
-      tc_fence_after();
-      bf16* out1 = p.dqkv + ((long)row_base + row) * dq + (KV ? vcol : h * HD);  // dV or dQ
-      bf16* out2 = p.dqkv + ((long)row_base + row) * dq + kcol;                  // dK
-      const float s1 = KV ? 1.f : p.scale;
+      if (ok && lane == 0) mbar_arrive(it_empty(rk % NR));
+      if (k < 0) break;
+      const BwdItem it = decode_item(p, k);
+      const int row = it.blk * 128 + r;  // key (KV) or query (Q) position of this thread
+      float lse_r = 0.f, d_r = 0.f;
+      if (!it.kv && row < p.T) {
+        const long o = ((long)it.b * p.H + it.head) * p.T + row;
+        lse_r = p.lse[o];
+        d_r = p.dvec[o];
+      }
+      for (int j = 0, jj = 0; j < it.nit; ++j, ++g) {
+        const int s = g % NS;
+        const int c0 = (it.kv ? it.blk + jj : jj) * 128 + 64 * half;  // first streamed position of this warp's columns
+        if (++jj == it.nit_h) jj = 0;
+        // causal / sequence-end mask needed anywhere in this warp's 64 x 32 piece?
+        const bool edge = it.kv ? (c0 < it.blk * 128 + 127 || c0 + 63 >= p.T || it.blk * 128 + 127 >= p.T)
+                                : (c0 + 63 > it.blk * 128 || c0 + 63 >= p.T || it.blk * 128 + 127 >= p.T);
+        if (!mbar_wait(s_full, g & 1, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        float sv[64];
+        TMEM_LD32(lane_addr + T_S + 64 * half, (reinterpret_cast<uint32_t*>(sv)));
+        TMEM_LD32(lane_addr + T_S + 64 * half + 32, (reinterpret_cast<uint32_t*>(sv) + 32));
+        if (it.kv) {
+          tmem_wait_ld();
+          if (!mbar_wait(st_full(s), (g / NS) & 1, abort_flag)) { ok = false; break; }
+          const float* vl = vec_base + s * 256 + 64 * half;   // lse / D of this warp's 64 queries
+          // P^T = 2^(S^T * scale - lse[q])
 #pragma unroll
-      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
-        uint32_t a[32], k[32];
-        TMEM_LD32(lane_addr + T_A1 + c, a);
-        if (KV) TMEM_LD32(lane_addr + T_A2 + c, k);
-        tmem_wait_ld();
-        if (row < p.T) {
+          for (int i = 0; i < 64; i += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(vl + i);
+            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
 #pragma unroll
-          for (int i = 0; i < 32; i += 8) {
-            uint4 v;
-            __nv_bfloat162 y0 = __floats2bfloat162_rn(__uint_as_float(a[i]) * s1, __uint_as_float(a[i + 1]) * s1);
-            __nv_bfloat162 y1 = __floats2bfloat162_rn(__uint_as_float(a[i + 2]) * s1, __uint_as_float(a[i + 3]) * s1);
-            __nv_bfloat162 y2 = __floats2bfloat162_rn(__uint_as_float(a[i + 4]) * s1, __uint_as_float(a[i + 5]) * s1);
-            __nv_bfloat162 y3 = __floats2bfloat162_rn(__uint_as_float(a[i + 6]) * s1, __uint_as_float(a[i + 7]) * s1);
-            v.x = *reinterpret_cast<uint32_t*>(&y0); v.y = *reinterpret_cast<uint32_t*>(&y1);
-            v.z = *reinterpret_cast<uint32_t*>(&y2); v.w = *reinterpret_cast<uint32_t*>(&y3);
-            *reinterpret_cast<uint4*>(out1 + c + i) = v;
-            if (KV) {
-              uint4 w;
-              __nv_bfloat162 x0 = __floats2bfloat162_rn(__uint_as_float(k[i]) * p.scale, __uint_as_float(k[i + 1]) * p.scale);
-              __nv_bfloat162 x1 = __floats2bfloat162_rn(__uint_as_float(k[i + 2]) * p.scale, __uint_as_float(k[i + 3]) * p.scale);
-              __nv_bfloat162 x2 = __floats2bfloat162_rn(__uint_as_float(k[i + 4]) * p.scale, __uint_as_float(k[i + 5]) * p.scale);
-              __nv_bfloat162 x3 = __floats2bfloat162_rn(__uint_as_float(k[i + 6]) * p.scale, __uint_as_float(k[i + 7]) * p.scale);
-              w.x = *reinterpret_cast<uint32_t*>(&x0); w.y = *reinterpret_cast<uint32_t*>(&x1);
-              w.z = *reinterpret_cast<uint32_t*>(&x2); w.w = *reinterpret_cast<uint32_t*>(&x3);
-              *reinterpret_cast<uint4*>(out2 + c + i) = w;
+            for (int e = 0; e < 4; ++e) {
+              const float a = fmaf(sv[i + e], sl2, -lv[e]);
+              float pe = ex2_approx(a);
+              if (edge) {
+                const int c = c0 + i + e;
+                if (c >= p.T || row >= p.T || c < row) pe = 0.f;
+              }
+              sv[i + e] = pe;
             }
           }
+          uint32_t pw[32];
+#pragma unroll
+          for (int w = 0; w < 32; ++w) {
+            __nv_bfloat162 t = __floats2bfloat162_rn(sv[2 * w], sv[2 * w + 1]);
+            pw[w] = *reinterpret_cast<uint32_t*>(&t);
+          }
+          TMEM_ST16(lane_addr + T_S + 64 * half, pw);
+          TMEM_ST16(lane_addr + T_S + 64 * half + 16, (pw + 16));
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(p_full);
+          // dS^T = P^T (dP^T - D[q]) in bf16 pairs over this warp's dP^T columns, 32 at a time
+          if (!mbar_wait(dp_full, g & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int hc = 0; hc < 2; ++hc) {
+            uint32_t dr[32];
+            TMEM_LD32(lane_addr + T_DP + 64 * half + 32 * hc, dr);
+            tmem_wait_ld();
+            uint32_t dw[16];
+#pragma unroll
+            for (int w = 0; w < 16; ++w) {
+              const int i = 32 * hc + 2 * w;
+              const float2 dd = *reinterpret_cast<const float2*>(vl + 128 + i);
+              __nv_bfloat162 t = __floats2bfloat162_rn(sv[i] * (__uint_as_float(dr[2 * w]) - dd.x),
+                                                       sv[i + 1] * (__uint_as_float(dr[2 * w + 1]) - dd.y));
+              dw[w] = *reinterpret_cast<uint32_t*>(&t);
+            }
+            TMEM_ST16(lane_addr + T_DP + 64 * half + 16 * hc, dw);
+          }
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(rd);
+            mbar_arrive(ds_full);
+          }
+          ++gk;
+        } else {
+          if (!mbar_wait(dp_full, g & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          float dv[64];
+          TMEM_LD32(lane_addr + T_DP + 64 * half, (reinterpret_cast<uint32_t*>(dv)));
+          TMEM_LD32(lane_addr + T_DP + 64 * half + 32, (reinterpret_cast<uint32_t*>(dv) + 32));
+          tmem_wait_ld();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(rd);  // S and dP of this block are in registers
+          const float nl = -lse_r;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) {
+            const float a = fmaf(sv[i], sl2, nl);
+            float pr = ex2_approx(a);
+            if (edge) {
+              const int c = c0 + i;
+              if (c >= p.T || row >= p.T || c > row) pr = 0.f;
+            }
+            dv[i] = pr * (dv[i] - d_r);
+          }
+          uint32_t dw[32];
+#pragma unroll
+          for (int w = 0; w < 32; ++w) {
+            __nv_bfloat162 t = __floats2bfloat162_rn(dv[2 * w], dv[2 * w + 1]);
+            dw[w] = *reinterpret_cast<uint32_t*>(&t);
+          }
+          // dS columns are free once the previous block's dQ (or dK) product has run
+          if (g > 0 && !mbar_wait(ds_empty, (g - 1) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          TMEM_ST16(lane_addr + T_DS + 32 * half, dw);
+          TMEM_ST16(lane_addr + T_DS + 32 * half + 16, (dw + 16));
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(ds_full);
         }
       }
-    } else if (lane == 0) {
-      set_dev_err(p.err, DEV_ERR_TIMEOUT);
+      if (!ok) break;
+      // ---------------------------------------------- epilogue: dK (scaled) and dV, or dQ (scaled)
+      // Each accumulator goes through the staging tile (bf16, 128-byte swizzle)
+      // and leaves by TMA stores into dqkv viewed as [B][T][dq], which clip the
+      // rows past the end of the sequence.
+      if (!mbar_wait(acc_full, n & 1, abort_flag)) { ok = false; break; }
+      tc_fence_after();
+      const int kcol = d + (it.kv ? it.head : it.head / gs) * HD;
+      const int nacc = it.kv ? 2 : 1;
+      for (int a = 0; a < nacc && ok; ++a, ++su) {
+        // accumulator a: dV (KV) / dQ (Q) from T_A1, then dK (KV) from T_A2
+        const uint32_t tcol = a ? T_A2 : T_A1;
+        const float sc = (it.kv && a == 0) ? 1.f : p.scale;
+        const int ocol = it.kv ? (a ? kcol : kcol + p.Hkv * HD) : it.head * HD;
+        uint32_t acc[HD / 2];
+        TMEM_LD32(lane_addr + tcol + half * (HD / 2), acc);
+        if constexpr (HD == 128) TMEM_LD32(lane_addr + tcol + half * (HD / 2) + 32, (acc + 32));
+        tmem_wait_ld();
+        if (a + 1 == nacc) {
+          // the accumulators are in registers: the next item's products may start
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(acc_empty);
+        }
+        // the staging tile is free once the previous TMA store has read it
+        if (!mbar_wait(stg_empty, (su & 1) ^ 1u, abort_flag)) { ok = false; break; }
+#pragma unroll
+        for (int u = 0; u < HD / 16; ++u) {
+          uint32_t w4[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 t = __floats2bfloat162_rn(__uint_as_float(acc[8 * u + 2 * e]) * sc,
+                                                     __uint_as_float(acc[8 * u + 2 * e + 1]) * sc);
+            w4[e] = *reinterpret_cast<uint32_t*>(&t);
+          }
+          *reinterpret_cast<uint4*>(stg_row + (((u0 + u) ^ (r & 7)) << 4)) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(stg_full);
+        if (storer) {
+          if (!mbar_wait(stg_full, su & 1, abort_flag)) { ok = false; break; }
+          for (int c = 0; c < KCH; ++c)
+            tma_store_3d(&p.dqkv_st, base + L::STG_OFF + c * L::CH, ocol + 64 * c, it.blk * 128, it.b);
+          bulk_commit();
+          bulk_wait_read_all();
+          mbar_arrive(stg_empty);
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      ++n;
     }
+    if (storer) bulk_wait_all();
+    if (!ok && lane == 0) set_dev_err(p.err, DEV_ERR_TIMEOUT);
   }
 
   tc_fence_before();
@@ -362,63 +592,95 @@ __device__ __forceinline__ void attn_bwd2_body(const AttnBwd2Params& p, int bx) 
   }
 }
 
-// Both passes in one launch (they read the same inputs and write disjoint
-// columns of dqkv): even x runs pass KV, odd x pass Q, so the heaviest blocks of
-// both go first and the two passes share one wave tail instead of two.
-template <int HD>
-__global__ void __launch_bounds__(AB2_THREADS, 1) attn_bwd2_kernel(const __grid_constant__ AttnBwd2Params p) {
-  if (blockIdx.x & 1) attn_bwd2_body<HD, false>(p, (int)(blockIdx.x >> 1));
-  else attn_bwd2_body<HD, true>(p, (int)(blockIdx.x >> 1));
+// 3-D bf16 tensor map (128-byte swizzle) over dqkv viewed as [B][T][dq], box
+// 64 x 128 x 1, for the epilogue's stores: rows past the end of a sequence are
+// clipped by the T extent instead of landing in the next sequence.
+bool dqkv_store_map(CUtensorMap* m, void* ptr, long dq, int T, int B, std::string* msg) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (!encode) {
+    if (msg) *msg = "cuTensorMapEncodeTiled not available from the driver";
+    return false;
+  }
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15) || ((dq * 2) & 15)) {
+    if (msg) *msg = "dqkv needs a 16-byte aligned base and a 16-byte multiple row pitch";
+    return false;
+  }
+  cuuint64_t dims[3] = {(cuuint64_t)dq, (cuuint64_t)T, (cuuint64_t)B};
+  cuuint64_t strides[2] = {(cuuint64_t)dq * 2, (cuuint64_t)dq * 2 * T};
+  cuuint32_t box[3] = {64, 128, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  if (encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+      CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (dqkv store map) failed";
+    return false;
+  }
+  return true;
 }
 
 template <int HD>
-int launch_bwd2(const AttnBwd2Params& p, int BH, cudaStream_t s, std::string* msg) {
-  constexpr int smem = Bwd2Smem<HD, true>::TOTAL > Bwd2Smem<HD, false>::TOTAL ? Bwd2Smem<HD, true>::TOTAL
-                                                                               : Bwd2Smem<HD, false>::TOTAL;
-  static_assert(smem <= 232448, "attention backward shared memory");
+int launch_bwd(const AttnBwdParams& p, cudaStream_t s, std::string* msg) {
+  constexpr int smem = BwdSmem<HD>::LAUNCH;
+  static_assert(BwdSmem<HD>::TOTAL + 512 <= smem, "attention backward shared memory");
   static bool set = false;
   if (!set) {
-    if (cudaFuncSetAttribute(attn_bwd2_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) {
+    if (cudaFuncSetAttribute(attn_bwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) {
       if (msg) *msg = "attention backward smem attribute failed";
       return 4;
     }
     set = true;
   }
-  dim3 grid(2 * p.nblk, BH);
-  attn_bwd2_kernel<HD><<<grid, AB2_THREADS, smem, s>>>(p);
+  const int total = p.nblk * p.B * (p.Hkv + p.H);
+  const int grid = total < num_sms() ? total : num_sms();
+  if (cudaMemsetAsync(p.next_item, 0, sizeof(int), s) != cudaSuccess) {
+    if (msg) *msg = "attention backward: clearing the work counter failed";
+    return 4;
+  }
+  attn_bwd_kernel<HD><<<grid, AB_THREADS, smem, s>>>(p);
   count_launches(1);
   return 0;
 }
 
 }  // namespace
 
-int attn_bwd2_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
-                 const float* dvec, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg) {
+int attn_bwd_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
+                const float* dvec, int* counter, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg) {
   if (B <= 0 || T <= 0) return 0;
   if (hd != 64 && hd != 128) { if (msg) *msg = "tcgen05 attention needs head_dim 64 or 128"; return 6; }
   if (Hkv <= 0 || H % Hkv) { if (msg) *msg = "heads must be a multiple of the key/value heads"; return 1; }
-  AttnBwd2Params p;
+  AttnBwdParams p;
   memset(&p, 0, sizeof(p));
   const long d = (long)H * hd, dq = (long)(H + 2 * Hkv) * hd;
   const unsigned long long rows = (unsigned long long)B * T;
-  if (!tma_map_2d(&p.qkv128, qkv, 0, dq, rows, dq, 64, 128, 1, msg) ||
-      !tma_map_2d(&p.qkv64, qkv, 0, dq, rows, dq, 64, 64, 1, msg) ||
-      !tma_map_2d(&p.do128, dctx, 0, d, rows, d, 64, 128, 1, msg) ||
-      !tma_map_2d(&p.do64, dctx, 0, d, rows, d, 64, 64, 1, msg))
+  if (!tma_map_2d(&p.qkv, qkv, 0, dq, rows, dq, 64, 128, 1, msg) || !tma_map_2d(&p.dout, dctx, 0, d, rows, d, 64, 128, 1, msg) ||
+      !dqkv_store_map(&p.dqkv_st, dqkv, dq, T, B, msg))
     return 1;
+  const long nblk = (T + 127) / 128;
+  if (nblk * B * (long)(Hkv + H) > 0x7fffffffL) { if (msg) *msg = "attention backward: too many work items"; return 1; }
   p.lse = lse;
   p.dvec = dvec;
   p.dqkv = reinterpret_cast<bf16*>(dqkv);
+  p.next_item = counter;
+  p.B = B;
   p.T = T;
   p.H = H;
   p.Hkv = Hkv;
-  p.nblk = (T + 127) / 128;
+  p.nblk = (int)nblk;
+  // bands of about eight query heads
+  const int gs = H / Hkv;
+  p.band = gs >= 8 ? 1 : 8 / gs;
   p.scale = 1.f / sqrtf((float)hd);
   p.scale_log2 = 1.4426950408889634f / sqrtf((float)hd);
   p.err = dev_err;
-  int r;
-  if (hd == 64) r = launch_bwd2<64>(p, B * H, s, msg);
-  else r = launch_bwd2<128>(p, B * H, s, msg);
+  const int r = hd == 64 ? launch_bwd<64>(p, s, msg) : launch_bwd<128>(p, s, msg);
   if (r) return r;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) { if (msg) *msg = std::string("attention backward launch: ") + cudaGetErrorString(e); return 4; }

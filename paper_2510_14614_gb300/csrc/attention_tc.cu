@@ -24,7 +24,7 @@
 
 #include "common.cuh"
 #include "internal.h"
-#include "tc_ptx.cuh"
+#include "attn_ptx.cuh"
 
 namespace fal {
 
@@ -152,6 +152,7 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
     // ------------------------------------------------ MMA issuer
     const uint32_t id_qk = make_idesc_bf16(0, 0, AT_BM, AT_BN);
     const uint32_t id_pv = make_idesc_bf16(0, 1, AT_BM, HD);
+    const uint32_t dhi = desc_hi(1024);
     bool ok = mbar_wait(qfull, 0, abort_flag);
     bool issued = false;
     // S_x = Q_x K_j^T into columns 128 x
@@ -160,12 +161,13 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
       if (!mbar_wait(kfull(s), (j >> 1) & 1, abort_flag)) return false;
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t qo = base + (x ? L::QB_OFF : L::QA_OFF);
+        // descriptor low words stepped by immediates along K (one shared high word)
+        const uint32_t lo_q = desc_lo(base + (x ? L::QB_OFF : L::QA_OFF), 16);
+        const uint32_t lo_k = desc_lo(base + L::K_OFF + s * KCH * L::CHUNK, 16);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint32_t qa = qo + (kk >> 2) * L::CHUNK + (kk & 3) * 32;
-          const uint32_t kb = base + L::K_OFF + (s * KCH + (kk >> 2)) * L::CHUNK + (kk & 3) * 32;
-          tc_mma(tmem + x * AT_BN, smem_desc(qa, 16, 1024), smem_desc(kb, 16, 1024), id_qk, kk > 0);
+          const uint32_t o = (kk >> 2) * (L::CHUNK >> 4) + (kk & 3) * 2;
+          tc_mma_w(tmem + x * AT_BN, lo_q + o, lo_k + o, dhi, id_qk, kk > 0);
         }
         tc_commit(sfull(x));
       }
@@ -180,12 +182,10 @@ __global__ void __launch_bounds__(AT2_THREADS, 1) attn_fwd2_kernel(const __grid_
       if (!mbar_wait(vfull(s), (j >> 1) & 1, abort_flag)) return false;
       tc_fence_after();
       if (lane == 0) {
+        const uint32_t lo_v = desc_lo(base + L::V_OFF + s * KCH * L::CHUNK, L::CHUNK);  // MN-major
 #pragma unroll
-        for (int kk = 0; kk < AT_BN / 16; ++kk) {
-          const uint32_t vb = base + L::V_OFF + s * KCH * L::CHUNK + kk * 2048;
-          tc_mma_ts(tmem + 256 + x * HD, tmem + x * AT_BN + kk * 8, smem_desc(vb, L::CHUNK, 1024), id_pv,
-                    (j > 0 || kk > 0));
-        }
+        for (int kk = 0; kk < AT_BN / 16; ++kk)
+          tc_mma_ts_w(tmem + 256 + x * HD, tmem + x * AT_BN + kk * 8, lo_v + kk * 128, dhi, id_pv, (j > 0 || kk > 0));
         tc_commit(odone(x));
       }
       __syncwarp();

@@ -92,8 +92,12 @@ constexpr int kCeSliceTc = 128, kCeSliceSimt = 64;
 // 0 means H (multi-head attention).
 int attn_fwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
              cudaStream_t s, std::string* msg, int Hkv = 0);
-// dvec: fp32 [B, H, T] scratch (receives D = rowsum(dO * O)); d_ready: dvec
+// dvec: fp32 scratch of attn_bwd_scratch_floats(B, T, H) floats: D = rowsum(dO * O)
+// in [B, H, T] layout, then the backward kernel's work counter; d_ready: dvec
 // already holds D (computed by the GEMM that produced dctx).
+inline size_t attn_bwd_scratch_floats(long B, long T, long H) {
+  return (size_t)((B * H * T + 63) / 64 * 64 + 64);
+}
 int attn_bwd(int act_bf16, int B, int T, int H, int hd, const void* qkv, const void* ctx,
              const float* lse, const void* dctx, void* dqkv, float* dvec, int* dev_err,
              cudaStream_t s, std::string* msg, int d_ready = 0, int Hkv = 0);
@@ -205,10 +209,12 @@ bool tma_map_2d(void* map128, const void* ptr, int f32, unsigned long long inner
 // multi-head attention), qkv rows of (H + 2 Hkv) * hd.
 int attn_fwd_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, void* ctx, float* lse, int* dev_err,
                 cudaStream_t s, std::string* msg);
-// Two-pass tcgen05 attention backward (dK/dV per key block, then dQ per query
-// block, all accumulated in TMEM; no dQ accumulator).  dvec = rowsum(dO * O).
-int attn_bwd2_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
-                 const float* dvec, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
+// tcgen05 attention backward: one persistent launch over key-block items
+// (dK, dV) and query-block items (dQ), each accumulated in TMEM (no atomics, no
+// fp32 dQ accumulator).  dvec = rowsum(dO * O); counter: one int of device
+// memory that the launch uses as its work counter (cleared on the stream first).
+int attn_bwd_tc(int B, int T, int H, int Hkv, int hd, const void* qkv, const void* dctx, const float* lse,
+                const float* dvec, int* counter, void* dqkv, int* dev_err, cudaStream_t s, std::string* msg);
 
 // Process-wide count of kernel launches made by the library.
 void count_launches(long long n);

@@ -47,7 +47,8 @@ int fal_kernel_attention_fwd(int B, int T, int H, int hd, const void* qkv, void*
 
 size_t fal_kernel_attention_bwd_scratch(int B, int T, int H, int hd) {
   (void)hd;
-  return (size_t)B * H * T;
+  if (B <= 0 || T <= 0 || H <= 0) return 64;
+  return fal::attn_bwd_scratch_floats(B, T, H);
 }
 
 int fal_kernel_attention_bwd(int B, int T, int H, int hd, const void* qkv, const void* ctx, const float* lse,

@@ -392,7 +392,7 @@ void carve(fal_handle* h, uint8_t* base) {
   h->dctx = b.take<uint8_t>(BT * d * a);
   h->dh = b.take<uint8_t>(BT * F * a);
   h->dqkv = b.take<uint8_t>(BT * h->DQ * a);
-  h->dvec = b.take<float>((size_t)h->B * h->H * h->T);
+  h->dvec = b.take<float>(attn_bwd_scratch_floats(h->B, h->T, h->H));
   const int cs_cols = h->DQ > h->F ? h->DQ : h->F;  // widest column reduction: b_qkv or b_up
   h->part0 = b.take<float>(colsum_partial_floats(cs_cols));
   h->part1 = b.take<float>(colsum_partial_floats(cs_cols));
