@@ -8,29 +8,33 @@
 //            of the group:
 //              S^T = K Q^T,  dP^T = V dO^T                       (TMEM)
 //              P^T = 2^(S^T*scale*log2e - lse[q]),  dS^T = P^T (dP^T - D[q])
-//              dV += P^T dO  (P^T from TMEM),  dK += dS^T Q  (dS^T from shared memory)
+//              dV += P^T dO,  dK += dS^T Q  (P^T and dS^T in bf16 from TMEM)
 //   Q item   (batch, query head, 128-query block): resident Q and dO; streams
 //            the 128-key blocks up to the diagonal, recomputes S, dP, P, dS
 //            row-wise and accumulates dQ += dS K (dS from TMEM).
 //
 // Every product has N = 128 (or N = head_dim), the shape the tensor pipe runs
-// at its full rate.  Each CTA (one per SM) walks a fixed list of items: items
-// are ranked heaviest first (by the number of streamed blocks, KV before Q at
-// equal count) and dealt to the CTAs in snake order.  Roles per CTA (320
-// threads):
-//   warp 0      producer: the resident tiles of each item once its
-//               predecessor's last S / dP product has read the old ones, then
-//               the streamed tiles through a ring of stages; for KV items also
-//               lse and D of each query block.
-//   warp 1      MMA issuer (one thread).  KV item, per block j:
-//               dV_j, S_{j+1}, dP_{j+1}, dK_j — the scores of block j+1 are
-//               computed while the elementwise warps finish block j.  Q item:
+// at its full rate.  Each CTA (one per SM) takes items from a launch-wide
+// counter; items are ranked in bands of about eight heads (so the CTAs working
+// at any time share those heads' Q, K, V and dO in L2), heaviest first within
+// a band.  Roles per CTA (576 threads):
+//   warp 0      producer: takes the next item and hands it to the other roles,
+//               loads the item's resident tiles once its predecessor's last S /
+//               dP product has read the old ones, then the streamed tiles
+//               through a ring of stages; for KV items also lse and D of each
+//               query block.
+//   warp 1      MMA issuer (one thread).  KV item, per block j: dV_j, S_{j+1},
+//               dK_j, dP_{j+1} (dS^T_j is written over the dP^T_j columns, which
+//               dP_{j+1} overwrites only after dK_j has read them).  Q item:
 //               S_{j+1}, dP_{j+1} as soon as the elementwise warps hold S_j and
 //               dP_j in registers, then dQ_j.  The next item's S_0 and dP_0 run
 //               while the elementwise warps store this item's accumulators.
-//   warps 2..9  elementwise, two warps per TMEM lane quadrant (64 of the 128
+//   warps 2..17 elementwise, four warps per TMEM lane quadrant (32 of the 128
 //               streamed columns each), then the item's epilogue: dK (scaled)
-//               and dV, or dQ (scaled), in bf16.
+//               and dV, or dQ (scaled), through a shared-memory staging tile and
+//               TMA stores.
+// Waiting warps sleep in the mbarrier (a suspend-time hint) rather than spin,
+// leaving their issue slots to the warps that compute.
 // TMEM (512 columns): S 0..127, dP 128..255, accumulators from 256 (dV | dK,
 // or dQ followed by the Q item's dS in bf16 pairs).
 // D = rowsum(dO * O) is an input: in the model it comes from the epilogue of the
@@ -53,7 +57,11 @@ namespace {
 
 using namespace ptx;
 
-constexpr int AB_THREADS = 320;
+// Elementwise warps per TMEM lane quadrant: each takes 128 / AB_EW of the
+// streamed block's columns.
+constexpr int AB_EW = 4;
+constexpr int AB_COLS = 128 / AB_EW;
+constexpr int AB_THREADS = 64 + 128 * AB_EW;
 
 struct AttnBwdParams {
   CUtensorMap qkv;            // [B*T, dq] bf16, dq = (H + 2 Hkv) hd, box 64 x 128, 128-byte swizzle
@@ -167,16 +175,16 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
     for (int s = 0; s < NS; ++s) { mbar_init(st_full(s), 2); mbar_init(st_empty(s), 1); }
     mbar_init(s_full, 1);
     mbar_init(dp_full, 1);
-    mbar_init(rd, 8);
-    mbar_init(p_full, 8);
-    mbar_init(ds_full, 8);
+    mbar_init(rd, 4 * AB_EW);
+    mbar_init(p_full, 4 * AB_EW);
+    mbar_init(ds_full, 4 * AB_EW);
     mbar_init(ds_empty, 1);
-    mbar_init(stg_full, 8);
+    mbar_init(stg_full, 4 * AB_EW);
     mbar_init(stg_empty, 1);
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 8);
+    mbar_init(acc_empty, 4 * AB_EW);
     mbar_init(drain, 1);
-    for (int i = 0; i < NR; ++i) { mbar_init(it_full(i), 1); mbar_init(it_empty(i), 9); }
+    for (int i = 0; i < NR; ++i) { mbar_init(it_full(i), 1); mbar_init(it_empty(i), 4 * AB_EW + 1); }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -193,7 +201,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
   // n-th item of this CTA as handed out by the producer (-1: no more work)
   auto next_item = [&](int n, bool& ok) -> int {
     const int i = n % NR;
-    if (!mbar_wait(it_full(i), (n / NR) & 1, abort_flag)) { ok = false; return -1; }
+    if (!mbar_wait_sleep(it_full(i), (n / NR) & 1, abort_flag)) { ok = false; return -1; }
     return ring[i];
   };
 
@@ -203,7 +211,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
     int g = 0, n = 0;  // streamed blocks and resident sets issued so far
     for (int r = 0; ok; ++r) {
       // take the next item from the launch-wide counter and hand it to the other roles
-      if (!mbar_wait(it_empty(r % NR), ((r / NR) & 1) ^ 1u, abort_flag)) { ok = false; break; }
+      if (!mbar_wait_sleep(it_empty(r % NR), ((r / NR) & 1) ^ 1u, abort_flag)) { ok = false; break; }
       int k = 0;
       if (lane == 0) {
         k = atomicAdd(p.next_item, 1);
@@ -218,7 +226,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       const int kcol = d + (it.kv ? it.head : it.head / gs) * HD;
       const int vcol = kcol + p.Hkv * HD;
       // resident tiles, once the previous item's last S / dP products have read the old ones
-      if (!mbar_wait(res_empty, (n & 1) ^ 1u, abort_flag)) { ok = false; break; }
+      if (!mbar_wait_sleep(res_empty, (n & 1) ^ 1u, abort_flag)) { ok = false; break; }
       if (lane == 0) {
         mbar_arrive_expect_tx(res_full, 2 * KCH * L::CH);
         for (int c = 0; c < KCH; ++c) {
@@ -235,7 +243,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       ++n;
       for (int j = 0, jj = 0, hq = it.kv ? it.head * gs : it.head; j < it.nit; ++j, ++g) {
         const int s = g % NS;
-        if (!mbar_wait(st_empty(s), ((g / NS) & 1) ^ 1u, abort_flag)) { ok = false; break; }
+        if (!mbar_wait_sleep(st_empty(s), ((g / NS) & 1) ^ 1u, abort_flag)) { ok = false; break; }
         const int c0 = (it.kv ? it.blk + jj : jj) * 128;   // first streamed row of the block
         const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
         if (lane == 0) {
@@ -304,12 +312,14 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           tc_mma_w(tmem + dst, lo_res + o, lo_st + o, hi, id_s, kk > 0);
         }
       };
-      // accumulate A (bf16 pairs in TMEM from column a_col: k at 64*(k/64) + (k%64)/2,
-      // or 32*(k/64) + (k%64)/2 when a_step is 32) times the stage half as MN-major B
+      // accumulate A (bf16 pairs in TMEM from column a_col, each elementwise warp's
+      // AB_COLS values of k packed at a_step * (k / AB_COLS) + (k % AB_COLS) / 2)
+      // times the stage half as MN-major B
+      constexpr int KPW = AB_COLS / 16;  // K16 steps per elementwise warp's columns
       auto issue_acc = [&](uint32_t dst, uint32_t a_col, uint32_t a_step, uint32_t lo_b, bool acc) {
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          tc_mma_ts_w(tmem + dst, tmem + a_col + a_step * (kk >> 2) + 8 * (kk & 3), lo_b + kk * 128, hi, id_acc,
+          tc_mma_ts_w(tmem + dst, tmem + a_col + a_step * (kk / KPW) + 8 * (kk % KPW), lo_b + kk * 128, hi, id_acc,
                       (acc || kk > 0));
       };
       for (int r = 0; ok; ++r) {
@@ -317,9 +327,9 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
         if (ok) mbar_arrive(it_empty(r % NR));
         if (k < 0) break;
         const BwdItem it = decode_item(p, k);
-        if (!mbar_wait(res_full, n & 1, abort_flag)) { ok = false; break; }
-        if (!mbar_wait(st_full(g % NS), (g / NS) & 1, abort_flag)) { ok = false; break; }
-        if (g > 0 && !mbar_wait(rd, (g - 1) & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait_sleep(res_full, n & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait_sleep(st_full(g % NS), (g / NS) & 1, abort_flag)) { ok = false; break; }
+        if (g > 0 && !mbar_wait_sleep(rd, (g - 1) & 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
         issue_sdp(T_S, lo_ra, g % NS, 0);
         tc_commit(s_full);
@@ -334,21 +344,21 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           const bool more = j + 1 < it.nit;
           if (it.kv) {
             // dV += P^T dO
-            if (!mbar_wait(p_full, gk & 1, abort_flag)) { ok = false; break; }
-            if (j == 0 && n > 0 && !mbar_wait(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
+            if (!mbar_wait_sleep(p_full, gk & 1, abort_flag)) { ok = false; break; }
+            if (j == 0 && n > 0 && !mbar_wait_sleep(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A1, T_S, 64, lo_h1, j > 0);
+            issue_acc(T_A1, T_S, AB_COLS, lo_h1, j > 0);
             if (more) {
               // S_{j+1} overwrites P^T_j, which the products above read first (in-order pipe)
-              if (!mbar_wait(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
               tc_fence_after();
               issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
               tc_commit(s_full);
             }
             // dK += dS^T Q   (dS^T in bf16 pairs over the dP^T columns)
-            if (!mbar_wait(ds_full, g & 1, abort_flag)) { ok = false; break; }
+            if (!mbar_wait_sleep(ds_full, g & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A2, T_DP, 64, lo_h0, j > 0);
+            issue_acc(T_A2, T_DP, AB_COLS, lo_h0, j > 0);
             tc_commit(ds_empty);
             tc_commit(st_empty(s));
             if (more) {
@@ -360,8 +370,8 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
             ++gk;
           } else {
             if (more) {
-              if (!mbar_wait(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
-              if (!mbar_wait(rd, g & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(rd, g & 1, abort_flag)) { ok = false; break; }
               tc_fence_after();
               issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
               tc_commit(s_full);
@@ -369,11 +379,11 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
               tc_commit(dp_full);
               if (j + 2 == it.nit) tc_commit(res_empty);
             }
-            // dQ += dS K   (dS in bf16 pairs from column T_DS)
-            if (!mbar_wait(ds_full, g & 1, abort_flag)) { ok = false; break; }
-            if (j == 0 && n > 0 && !mbar_wait(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
+            // dQ += dS K   (dS in bf16 pairs from column T_DS, AB_COLS / 2 columns per warp)
+            if (!mbar_wait_sleep(ds_full, g & 1, abort_flag)) { ok = false; break; }
+            if (j == 0 && n > 0 && !mbar_wait_sleep(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A1, T_DS, 32, lo_h0, j > 0);
+            issue_acc(T_A1, T_DS, AB_COLS / 2, lo_h0, j > 0);
             tc_commit(ds_empty);
             tc_commit(st_empty(s));
           }
@@ -393,18 +403,20 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------ elementwise (two warps per lane quadrant)
-    const int q4 = warp & 3, half = (warp - 2) >> 2;
+    // ------------------------------------------------ elementwise (AB_EW warps per lane quadrant)
+    constexpr int C = AB_COLS;
+    const int q4 = warp & 3, part = (warp - 2) >> 2;
     const int r = q4 * 32 + lane;  // TMEM lane = row inside the 128-row block
     const uint32_t lane_addr = tmem + ((uint32_t)(q4 * 32) << 16);
     const float sl2 = p.scale_log2;
     const bool storer = warp == 2 && lane == 0;  // issues the epilogue's TMA stores
     bool ok = true;
     int g = 0, gk = 0, n = 0, su = 0;  // su: uses of the epilogue staging buffer
-    // this thread's part of a row of the staging tile (128-byte swizzle): head_dim
-    // 128: all of chunk `half`; head_dim 64: half of the one chunk
-    uint8_t* stg_row = sbase + L::STG_OFF + (HD == 128 ? half * L::CH : 0) + (r >> 3) * 1024 + (r & 7) * 128;
-    const int u0 = HD == 128 ? 0 : 4 * half;
+    // this thread's HD / AB_EW accumulator columns in its row of the staging tile
+    // (128-byte swizzle, 64-column chunks)
+    constexpr int EC = HD / AB_EW;
+    uint8_t* stg_row = sbase + L::STG_OFF + (part * EC / 64) * L::CH + (r >> 3) * 1024 + (r & 7) * 128;
+    const int u0 = (part * EC % 64) / 8;
     for (int rk = 0; ok; ++rk) {
       const int k = next_item(rk, ok);
       __syncwarp();
@@ -420,29 +432,28 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       }
       for (int j = 0, jj = 0; j < it.nit; ++j, ++g) {
         const int s = g % NS;
-        const int c0 = (it.kv ? it.blk + jj : jj) * 128 + 64 * half;  // first streamed position of this warp's columns
+        const int c0 = (it.kv ? it.blk + jj : jj) * 128 + C * part;  // first streamed position of this warp's columns
         if (++jj == it.nit_h) jj = 0;
-        // causal / sequence-end mask needed anywhere in this warp's 64 x 32 piece?
-        const bool edge = it.kv ? (c0 < it.blk * 128 + 127 || c0 + 63 >= p.T || it.blk * 128 + 127 >= p.T)
-                                : (c0 + 63 > it.blk * 128 || c0 + 63 >= p.T || it.blk * 128 + 127 >= p.T);
-        if (!mbar_wait(s_full, g & 1, abort_flag)) { ok = false; break; }
+        // causal / sequence-end mask needed anywhere in this warp's 32 x C piece?
+        const bool edge = it.kv ? (c0 < it.blk * 128 + 127 || c0 + C - 1 >= p.T || it.blk * 128 + 127 >= p.T)
+                                : (c0 + C - 1 > it.blk * 128 || c0 + C - 1 >= p.T || it.blk * 128 + 127 >= p.T);
+        if (!mbar_wait_sleep(s_full, g & 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        float sv[64];
-        TMEM_LD32(lane_addr + T_S + 64 * half, (reinterpret_cast<uint32_t*>(sv)));
-        TMEM_LD32(lane_addr + T_S + 64 * half + 32, (reinterpret_cast<uint32_t*>(sv) + 32));
+        float sv[C];
+#pragma unroll
+        for (int c = 0; c < C; c += 32) TMEM_LD32(lane_addr + T_S + C * part + c, (reinterpret_cast<uint32_t*>(sv) + c));
         if (it.kv) {
           tmem_wait_ld();
-          if (!mbar_wait(st_full(s), (g / NS) & 1, abort_flag)) { ok = false; break; }
-          const float* vl = vec_base + s * 256 + 64 * half;   // lse / D of this warp's 64 queries
+          if (!mbar_wait_sleep(st_full(s), (g / NS) & 1, abort_flag)) { ok = false; break; }
+          const float* vl = vec_base + s * 256 + C * part;   // lse / D of this warp's C queries
           // P^T = 2^(S^T * scale - lse[q])
 #pragma unroll
-          for (int i = 0; i < 64; i += 4) {
+          for (int i = 0; i < C; i += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(vl + i);
             const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const float a = fmaf(sv[i + e], sl2, -lv[e]);
-              float pe = ex2_approx(a);
+              float pe = ex2_approx(fmaf(sv[i + e], sl2, -lv[e]));
               if (edge) {
                 const int c = c0 + i + e;
                 if (c >= p.T || row >= p.T || c < row) pe = 0.f;
@@ -450,25 +461,26 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
               sv[i + e] = pe;
             }
           }
-          uint32_t pw[32];
+          // P^T in bf16 pairs over the first C / 2 of this warp's S^T columns
+          uint32_t pw[C / 2];
 #pragma unroll
-          for (int w = 0; w < 32; ++w) {
+          for (int w = 0; w < C / 2; ++w) {
             __nv_bfloat162 t = __floats2bfloat162_rn(sv[2 * w], sv[2 * w + 1]);
             pw[w] = *reinterpret_cast<uint32_t*>(&t);
           }
-          TMEM_ST16(lane_addr + T_S + 64 * half, pw);
-          TMEM_ST16(lane_addr + T_S + 64 * half + 16, (pw + 16));
+#pragma unroll
+          for (int c = 0; c < C / 2; c += 16) TMEM_ST16(lane_addr + T_S + C * part + c, (pw + c));
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(p_full);
           // dS^T = P^T (dP^T - D[q]) in bf16 pairs over this warp's dP^T columns, 32 at a time
-          if (!mbar_wait(dp_full, g & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_sleep(dp_full, g & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
-          for (int hc = 0; hc < 2; ++hc) {
+          for (int hc = 0; hc < C / 32; ++hc) {
             uint32_t dr[32];
-            TMEM_LD32(lane_addr + T_DP + 64 * half + 32 * hc, dr);
+            TMEM_LD32(lane_addr + T_DP + C * part + 32 * hc, dr);
             tmem_wait_ld();
             uint32_t dw[16];
 #pragma unroll
@@ -479,7 +491,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
                                                        sv[i + 1] * (__uint_as_float(dr[2 * w + 1]) - dd.y));
               dw[w] = *reinterpret_cast<uint32_t*>(&t);
             }
-            TMEM_ST16(lane_addr + T_DP + 64 * half + 16 * hc, dw);
+            TMEM_ST16(lane_addr + T_DP + C * part + 16 * hc, dw);
           }
           tmem_wait_st();
           tc_fence_before();
@@ -490,37 +502,36 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           }
           ++gk;
         } else {
-          if (!mbar_wait(dp_full, g & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_sleep(dp_full, g & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          float dv[64];
-          TMEM_LD32(lane_addr + T_DP + 64 * half, (reinterpret_cast<uint32_t*>(dv)));
-          TMEM_LD32(lane_addr + T_DP + 64 * half + 32, (reinterpret_cast<uint32_t*>(dv) + 32));
+          float dv[C];
+#pragma unroll
+          for (int c = 0; c < C; c += 32) TMEM_LD32(lane_addr + T_DP + C * part + c, (reinterpret_cast<uint32_t*>(dv) + c));
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(rd);  // S and dP of this block are in registers
           const float nl = -lse_r;
 #pragma unroll
-          for (int i = 0; i < 64; ++i) {
-            const float a = fmaf(sv[i], sl2, nl);
-            float pr = ex2_approx(a);
+          for (int i = 0; i < C; ++i) {
+            float pr = ex2_approx(fmaf(sv[i], sl2, nl));
             if (edge) {
               const int c = c0 + i;
               if (c >= p.T || row >= p.T || c > row) pr = 0.f;
             }
             dv[i] = pr * (dv[i] - d_r);
           }
-          uint32_t dw[32];
+          uint32_t dw[C / 2];
 #pragma unroll
-          for (int w = 0; w < 32; ++w) {
+          for (int w = 0; w < C / 2; ++w) {
             __nv_bfloat162 t = __floats2bfloat162_rn(dv[2 * w], dv[2 * w + 1]);
             dw[w] = *reinterpret_cast<uint32_t*>(&t);
           }
           // dS columns are free once the previous block's dQ (or dK) product has run
-          if (g > 0 && !mbar_wait(ds_empty, (g - 1) & 1, abort_flag)) { ok = false; break; }
+          if (g > 0 && !mbar_wait_sleep(ds_empty, (g - 1) & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          TMEM_ST16(lane_addr + T_DS + 32 * half, dw);
-          TMEM_ST16(lane_addr + T_DS + 32 * half + 16, (dw + 16));
+#pragma unroll
+          for (int c = 0; c < C / 2; c += 16) TMEM_ST16(lane_addr + T_DS + (C / 2) * part + c, (dw + c));
           tmem_wait_st();
           tc_fence_before();
           __syncwarp();
@@ -532,7 +543,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       // Each accumulator goes through the staging tile (bf16, 128-byte swizzle)
       // and leaves by TMA stores into dqkv viewed as [B][T][dq], which clip the
       // rows past the end of the sequence.
-      if (!mbar_wait(acc_full, n & 1, abort_flag)) { ok = false; break; }
+      if (!mbar_wait_sleep(acc_full, n & 1, abort_flag)) { ok = false; break; }
       tc_fence_after();
       const int kcol = d + (it.kv ? it.head : it.head / gs) * HD;
       const int nacc = it.kv ? 2 : 1;
@@ -541,9 +552,13 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
         const uint32_t tcol = a ? T_A2 : T_A1;
         const float sc = (it.kv && a == 0) ? 1.f : p.scale;
         const int ocol = it.kv ? (a ? kcol : kcol + p.Hkv * HD) : it.head * HD;
-        uint32_t acc[HD / 2];
-        TMEM_LD32(lane_addr + tcol + half * (HD / 2), acc);
-        if constexpr (HD == 128) TMEM_LD32(lane_addr + tcol + half * (HD / 2) + 32, (acc + 32));
+        uint32_t acc[EC];
+        if constexpr (EC >= 32) {
+#pragma unroll
+          for (int c = 0; c < EC; c += 32) TMEM_LD32(lane_addr + tcol + part * EC + c, (acc + c));
+        } else {
+          TMEM_LD16(lane_addr + tcol + part * EC, acc);
+        }
         tmem_wait_ld();
         if (a + 1 == nacc) {
           // the accumulators are in registers: the next item's products may start
@@ -552,9 +567,9 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           if (lane == 0) mbar_arrive(acc_empty);
         }
         // the staging tile is free once the previous TMA store has read it
-        if (!mbar_wait(stg_empty, (su & 1) ^ 1u, abort_flag)) { ok = false; break; }
+        if (!mbar_wait_sleep(stg_empty, (su & 1) ^ 1u, abort_flag)) { ok = false; break; }
 #pragma unroll
-        for (int u = 0; u < HD / 16; ++u) {
+        for (int u = 0; u < EC / 8; ++u) {
           uint32_t w4[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -568,7 +583,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
         __syncwarp();
         if (lane == 0) mbar_arrive(stg_full);
         if (storer) {
-          if (!mbar_wait(stg_full, su & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_sleep(stg_full, su & 1, abort_flag)) { ok = false; break; }
           for (int c = 0; c < KCH; ++c)
             tma_store_3d(&p.dqkv_st, base + L::STG_OFF + c * L::CH, ocol + 64 * c, it.blk * 128, it.b);
           bulk_commit();

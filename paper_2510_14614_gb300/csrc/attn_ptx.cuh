@@ -9,6 +9,30 @@
 namespace fal {
 namespace ptx {
 
+// Bounded mbarrier wait whose polls suspend the thread in hardware until the
+// phase completes (or 20 us pass), so that waiting warps leave their issue
+// slots to the warps that compute.  Same contract as mbar_wait: false if the
+// phase did not complete within kWaitNs or another role already gave up.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(20000u)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity, volatile uint32_t* abort_flag) {
+  if (mbar_try_wait_sleep(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait_sleep(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > kWaitNs) { *abort_flag = 1; return false; }
+  }
+}
+
 // High word of a tcgen05 shared-memory descriptor: stride byte offset >> 4,
 // version 1 (bit 46 of the descriptor), 128-byte swizzle (bits 61-63 = 2).
 __device__ __forceinline__ uint32_t desc_hi(uint32_t sbo) {
@@ -36,6 +60,15 @@ __device__ __forceinline__ void tc_mma_ts_w(uint32_t d_tmem, uint32_t a_tmem, ui
       "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(accum), "r"(idesc)
       : "memory");
 }
+// TMEM load, 32 lanes x 16 columns (one register per column).
+#define TMEM_LD16(taddr, r)                                                                          \
+  asm volatile(                                                                                      \
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];" \
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),          \
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),       \
+        "=r"(r[14]), "=r"(r[15])                                                                      \
+      : "r"(taddr))
+
 // TMA store of a shared-memory tile to global memory through a 3-D tensor map.
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int x, int y, int z) {
   asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
