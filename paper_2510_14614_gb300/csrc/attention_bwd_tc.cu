@@ -450,15 +450,17 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
 #pragma unroll
           for (int i = 0; i < C; i += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(vl + i);
-            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
+            sv[i] = ex2_approx(fmaf(sv[i], sl2, -l4.x));
+            sv[i + 1] = ex2_approx(fmaf(sv[i + 1], sl2, -l4.y));
+            sv[i + 2] = ex2_approx(fmaf(sv[i + 2], sl2, -l4.z));
+            sv[i + 3] = ex2_approx(fmaf(sv[i + 3], sl2, -l4.w));
+          }
+          if (edge) {
+            // causal mask (query c sees key row iff c >= row) and sequence ends
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              float pe = ex2_approx(fmaf(sv[i + e], sl2, -lv[e]));
-              if (edge) {
-                const int c = c0 + i + e;
-                if (c >= p.T || row >= p.T || c < row) pe = 0.f;
-              }
-              sv[i + e] = pe;
+            for (int i = 0; i < C; ++i) {
+              const int c = c0 + i;
+              if (c >= p.T || row >= p.T || c < row) sv[i] = 0.f;
             }
           }
           // P^T in bf16 pairs over the first C / 2 of this warp's S^T columns
@@ -513,14 +515,17 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           if (lane == 0) mbar_arrive(rd);  // S and dP of this block are in registers
           const float nl = -lse_r;
 #pragma unroll
-          for (int i = 0; i < C; ++i) {
-            float pr = ex2_approx(fmaf(sv[i], sl2, nl));
-            if (edge) {
+          for (int i = 0; i < C; ++i) sv[i] = ex2_approx(fmaf(sv[i], sl2, nl));
+          if (edge) {
+            // causal mask (key c visible to query row iff c <= row) and sequence ends
+#pragma unroll
+            for (int i = 0; i < C; ++i) {
               const int c = c0 + i;
-              if (c >= p.T || row >= p.T || c > row) pr = 0.f;
+              if (c >= p.T || row >= p.T || c > row) sv[i] = 0.f;
             }
-            dv[i] = pr * (dv[i] - d_r);
           }
+#pragma unroll
+          for (int i = 0; i < C; ++i) dv[i] = sv[i] * (dv[i] - d_r);
           uint32_t dw[C / 2];
 #pragma unroll
           for (int w = 0; w < C / 2; ++w) {
