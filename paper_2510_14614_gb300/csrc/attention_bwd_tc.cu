@@ -21,14 +21,18 @@
 //   warp 0      producer: takes the next item and hands it to the other roles,
 //               loads the item's resident tiles once its predecessor's last S /
 //               dP product has read the old ones, then the streamed tiles
-//               through a ring of stages; for KV items also lse and D of each
-//               query block.
+//               through a ring of stages whose two halves are filled and freed
+//               separately, their roles alternating with every use; for KV
+//               items also lse and D of each query block.
 //   warp 1      MMA issuer (one thread).  KV item, per block j: dV_j, S_{j+1},
 //               dK_j, dP_{j+1} (dS^T_j is written over the dP^T_j columns, which
 //               dP_{j+1} overwrites only after dK_j has read them).  Q item:
-//               S_{j+1}, dP_{j+1} as soon as the elementwise warps hold S_j and
-//               dP_j in registers, then dQ_j.  The next item's S_0 and dP_0 run
-//               while the elementwise warps store this item's accumulators.
+//               S_{j+1} as soon as the elementwise warps hold S_j in registers,
+//               dQ_j, then dP_{j+1} (head_dim 128, two stages: the K block of
+//               j+2 loads into the half V_j leaves after dP_j, so S_{j+2} need
+//               not wait for dQ_j); with four stages dP_{j+1} precedes dQ_j.
+//               The next item's S_0 and dP_0 run while the elementwise warps
+//               store this item's accumulators.
 //   warps 2..17 elementwise, four warps per TMEM lane quadrant (32 of the 128
 //               streamed columns each), then the item's epilogue: dK (scaled)
 //               and dV, or dQ (scaled), through a shared-memory staging tile and
@@ -90,7 +94,7 @@ struct BwdSmem {
   static constexpr int STG_OFF = ST_OFF + STAGES * STAGE;  // epilogue staging: one accumulator in bf16
   static constexpr int VEC_OFF = STG_OFF + KCH * CH;   // lse[128] | D[128] per stage (KV items)
   static constexpr int BAR_OFF = VEC_OFF + STAGES * 1024;
-  static constexpr int TOTAL = BAR_OFF + 256;
+  static constexpr int TOTAL = BAR_OFF + (HD == 64 ? 512 : 256);  // barriers, TMEM slot, item ring
   static constexpr int LAUNCH = TOTAL + 1024 < 232448 ? TOTAL + 1024 : 232448;  // + alignment slack
 };
 
@@ -139,7 +143,7 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
 template <int HD>
 __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_constant__ AttnBwdParams p) {
   using L = BwdSmem<HD>;
-  constexpr int KCH = L::KCH, NS = L::STAGES, NR = 4;
+  constexpr int KCH = L::KCH, NS = L::STAGES, NR = 2;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -151,14 +155,21 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
   uint8_t* sbase = smem_raw + (base - raw);
   const uint32_t bar = base + L::BAR_OFF;
   const uint32_t res_full = bar, res_empty = bar + 8;
-  auto st_full = [&](int s) { return bar + 8u * (2 + s); };
-  auto st_empty = [&](int s) { return bar + 8u * (2 + NS + s); };
-  const uint32_t s_full = bar + 8u * (2 + 2 * NS), dp_full = s_full + 8, rd = s_full + 16, p_full = s_full + 24,
-                 ds_full = s_full + 32, ds_empty = s_full + 40, stg_full = s_full + 48, stg_empty = s_full + 56,
-                 acc_full = s_full + 64, acc_empty = s_full + 72, drain = s_full + 80;
-  auto it_full = [&](int i) { return s_full + 88 + 8u * i; };
-  auto it_empty = [&](int i) { return s_full + 88 + 8u * (NR + i); };
-  uint8_t* misc = sbase + L::BAR_OFF + 8 * (13 + 2 * NS + 2 * NR);
+  // Each stage has two halves with their own barriers.  Streamed block g uses
+  // stage g % NS; its first operand (Q of a KV block, K of a Q block) goes into
+  // half ha(g) = (g / NS) & 1 and its second (dO, V) into the other half, so the
+  // roles alternate on every use of a stage: a Q block's V half, free once dP has
+  // read it, takes the K of the block two later, whose S product is needed soon,
+  // while the K half, free only after dQ, takes its V.
+  auto hf_full = [&](int s, int hh) { return bar + 8u * (2 + 2 * s + hh); };
+  auto hf_empty = [&](int s, int hh) { return bar + 8u * (2 + 2 * NS + 2 * s + hh); };
+  auto ha_of = [&](int g) { return (g / NS) & 1; };
+  const uint32_t s_full = bar + 8u * (2 + 4 * NS), dp_full = s_full + 8, rd_s = s_full + 16, rd_dp = s_full + 24,
+                 p_full = s_full + 32, ds_full = s_full + 40, ds_empty = s_full + 48, stg_full = s_full + 56,
+                 stg_empty = s_full + 64, acc_full = s_full + 72, acc_empty = s_full + 80, drain = s_full + 88;
+  auto it_full = [&](int i) { return s_full + 96 + 8u * i; };
+  auto it_empty = [&](int i) { return s_full + 96 + 8u * (NR + i); };
+  uint8_t* misc = sbase + L::BAR_OFF + 8 * (14 + 4 * NS + 2 * NR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc);
   volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(misc + 4);
   volatile int* ring = reinterpret_cast<volatile int*>(misc + 8);  // item ranks handed from the producer to the other roles
@@ -172,10 +183,12 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
   if (threadIdx.x == 0) {
     mbar_init(res_full, 1);
     mbar_init(res_empty, 1);
-    for (int s = 0; s < NS; ++s) { mbar_init(st_full(s), 2); mbar_init(st_empty(s), 1); }
+    for (int s = 0; s < NS; ++s)
+      for (int hh = 0; hh < 2; ++hh) { mbar_init(hf_full(s, hh), 2); mbar_init(hf_empty(s, hh), 1); }
     mbar_init(s_full, 1);
     mbar_init(dp_full, 1);
-    mbar_init(rd, 4 * AB_EW);
+    mbar_init(rd_s, 4 * AB_EW);
+    mbar_init(rd_dp, 4 * AB_EW);
     mbar_init(p_full, 4 * AB_EW);
     mbar_init(ds_full, 4 * AB_EW);
     mbar_init(ds_empty, 1);
@@ -241,45 +254,46 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       }
       __syncwarp();
       ++n;
-      for (int j = 0, jj = 0, hq = it.kv ? it.head * gs : it.head; j < it.nit; ++j, ++g) {
-        const int s = g % NS;
-        if (!mbar_wait_sleep(st_empty(s), ((g / NS) & 1) ^ 1u, abort_flag)) { ok = false; break; }
+      for (int j = 0, jj = 0, hq = it.kv ? it.head * gs : it.head; j < it.nit && ok; ++j, ++g) {
+        const int s = g % NS, ha = ha_of(g);
+        const uint32_t par = ((g / NS) & 1) ^ 1u;
         const int c0 = (it.kv ? it.blk + jj : jj) * 128;   // first streamed row of the block
         const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
-        if (lane == 0) {
-          mbar_arrive_expect_tx(st_full(s), L::STAGE);
-          for (int c = 0; c < KCH; ++c) {
-            if (it.kv) {
-              tma_load_2d(sb + c * L::CH, &p.qkv, hq * HD + 64 * c, row_base + c0, st_full(s));
-              tma_load_2d(sb + L::HALF + c * L::CH, &p.dout, hq * HD + 64 * c, row_base + c0, st_full(s));
-            } else {
-              tma_load_2d(sb + c * L::CH, &p.qkv, kcol + 64 * c, row_base + c0, st_full(s));
-              tma_load_2d(sb + L::HALF + c * L::CH, &p.qkv, vcol + 64 * c, row_base + c0, st_full(s));
+        for (int t = 0; t < 2; ++t) {
+          // t = 0: Q (KV) or K (Q) into half ha; t = 1: dO or V into the other half
+          const int hh = ha ^ t;
+          if (!mbar_wait_sleep(hf_empty(s, hh), par, abort_flag)) { ok = false; break; }
+          if (lane == 0) {
+            mbar_arrive_expect_tx(hf_full(s, hh), L::HALF);
+            for (int c = 0; c < KCH; ++c) {
+              const uint32_t dst = sb + hh * L::HALF + c * L::CH;
+              if (it.kv) tma_load_2d(dst, t ? &p.dout : &p.qkv, hq * HD + 64 * c, row_base + c0, hf_full(s, hh));
+              else tma_load_2d(dst, &p.qkv, (t ? vcol : kcol) + 64 * c, row_base + c0, hf_full(s, hh));
             }
           }
-        }
-        if (it.kv) {
-          // lse and D of the block's 128 queries (zero beyond the sequence): all
-          // eight loads of a lane are in flight together
-          float* v = reinterpret_cast<float*>(sbase + L::VEC_OFF + s * 1024);
-          const float* lsrc = p.lse + ((long)it.b * p.H + hq) * p.T;
-          const float* dsrc = p.dvec + ((long)it.b * p.H + hq) * p.T;
-          float lv[4], dvv[4];
+          if (it.kv && t == 0) {
+            // lse and D of the block's 128 queries (zero beyond the sequence): all
+            // eight loads of a lane are in flight together
+            float* v = reinterpret_cast<float*>(sbase + L::VEC_OFF + s * 1024);
+            const float* lsrc = p.lse + ((long)it.b * p.H + hq) * p.T;
+            const float* dsrc = p.dvec + ((long)it.b * p.H + hq) * p.T;
+            float lv[4], dvv[4];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int t = c0 + lane + 32 * q;
-            lv[q] = t < p.T ? __ldg(lsrc + t) : 0.f;
-            dvv[q] = t < p.T ? __ldg(dsrc + t) : 0.f;
-          }
+            for (int q = 0; q < 4; ++q) {
+              const int tt = c0 + lane + 32 * q;
+              lv[q] = tt < p.T ? __ldg(lsrc + tt) : 0.f;
+              dvv[q] = tt < p.T ? __ldg(dsrc + tt) : 0.f;
+            }
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            v[lane + 32 * q] = lv[q];
-            v[128 + lane + 32 * q] = dvv[q];
+            for (int q = 0; q < 4; ++q) {
+              v[lane + 32 * q] = lv[q];
+              v[128 + lane + 32 * q] = dvv[q];
+            }
           }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(hf_full(s, hh));
+          __syncwarp();
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(st_full(s));
-        __syncwarp();
         if (++jj == it.nit_h) { jj = 0; ++hq; }
       }
     }
@@ -289,7 +303,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       if (n > 0) drain_wait(res_full, (uint32_t)((n - 1) & 1));
       for (int s = 0; s < NS && s < g; ++s) {
         const int last = g - 1 - ((g - 1 - s) % NS);      // last block that used stage s
-        drain_wait(st_full(s), (uint32_t)((last / NS) & 1));
+        for (int hh = 0; hh < 2; ++hh) drain_wait(hf_full(s, hh), (uint32_t)((last / NS) & 1));
       }
     }
   } else if (warp == 1) {
@@ -328,64 +342,95 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
         if (k < 0) break;
         const BwdItem it = decode_item(p, k);
         if (!mbar_wait_sleep(res_full, n & 1, abort_flag)) { ok = false; break; }
-        if (!mbar_wait_sleep(st_full(g % NS), (g / NS) & 1, abort_flag)) { ok = false; break; }
-        if (g > 0 && !mbar_wait_sleep(rd, (g - 1) & 1, abort_flag)) { ok = false; break; }
-        tc_fence_after();
-        issue_sdp(T_S, lo_ra, g % NS, 0);
-        tc_commit(s_full);
-        issue_sdp(T_DP, lo_rb, g % NS, 1);
-        tc_commit(dp_full);
-        issued = true;
-        if (it.nit == 1) tc_commit(res_empty);
+        {
+          // S and dP of the item's first block: the S / dP columns are free once the
+          // elementwise warps have read the previous block's
+          const int s0 = g % NS, h0 = ha_of(g);
+          const uint32_t par0 = (g / NS) & 1;
+          if (!mbar_wait_sleep(hf_full(s0, h0), par0, abort_flag)) { ok = false; break; }
+          if (g > 0 && !mbar_wait_sleep(rd_s, (g - 1) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          issue_sdp(T_S, lo_ra, s0, h0);
+          tc_commit(s_full);
+          if (!mbar_wait_sleep(hf_full(s0, h0 ^ 1), par0, abort_flag)) { ok = false; break; }
+          if (g > 0 && !mbar_wait_sleep(rd_dp, (g - 1) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          issue_sdp(T_DP, lo_rb, s0, h0 ^ 1);
+          tc_commit(dp_full);
+          if (!it.kv) tc_commit(hf_empty(s0, h0 ^ 1));  // a Q block's V half: free once dP has read it
+          issued = true;
+          if (it.nit == 1) tc_commit(res_empty);
+        }
         for (int j = 0; j < it.nit; ++j, ++g) {
-          const int s = g % NS;
+          const int s = g % NS, ha = ha_of(g);
           const uint32_t sb = base + L::ST_OFF + s * L::STAGE;
-          const uint32_t lo_h0 = desc_lo(sb, L::CH), lo_h1 = desc_lo(sb + L::HALF, L::CH);  // MN-major B
+          // MN-major B descriptors of this block's two operands (first: Q or K, second: dO or V)
+          const uint32_t lo_first = desc_lo(sb + ha * L::HALF, L::CH), lo_second = desc_lo(sb + (ha ^ 1) * L::HALF, L::CH);
           const bool more = j + 1 < it.nit;
+          const int s1 = (g + 1) % NS, h1 = ha_of(g + 1);
+          const uint32_t par1 = ((g + 1) / NS) & 1;
           if (it.kv) {
             // dV += P^T dO
             if (!mbar_wait_sleep(p_full, gk & 1, abort_flag)) { ok = false; break; }
             if (j == 0 && n > 0 && !mbar_wait_sleep(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A1, T_S, AB_COLS, lo_h1, j > 0);
+            issue_acc(T_A1, T_S, AB_COLS, lo_second, j > 0);
             if (more) {
               // S_{j+1} overwrites P^T_j, which the products above read first (in-order pipe)
-              if (!mbar_wait_sleep(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(hf_full(s1, h1), par1, abort_flag)) { ok = false; break; }
               tc_fence_after();
-              issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
+              issue_sdp(T_S, lo_ra, s1, h1);
               tc_commit(s_full);
             }
             // dK += dS^T Q   (dS^T in bf16 pairs over the dP^T columns)
             if (!mbar_wait_sleep(ds_full, g & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A2, T_DP, AB_COLS, lo_h0, j > 0);
+            issue_acc(T_A2, T_DP, AB_COLS, lo_first, j > 0);
             tc_commit(ds_empty);
-            tc_commit(st_empty(s));
+            tc_commit(hf_empty(s, ha));
+            tc_commit(hf_empty(s, ha ^ 1));
             if (more) {
               // dP_{j+1} overwrites dS^T_j after the product above has read it
-              issue_sdp(T_DP, lo_rb, (g + 1) % NS, 1);
+              if (!mbar_wait_sleep(hf_full(s1, h1 ^ 1), par1, abort_flag)) { ok = false; break; }
+              tc_fence_after();
+              issue_sdp(T_DP, lo_rb, s1, h1 ^ 1);
               tc_commit(dp_full);
               if (j + 2 == it.nit) tc_commit(res_empty);
             }
             ++gk;
           } else {
+            // S_{j+1} as soon as its K block is in and S_j has been read; dP_{j+1}
+            // once its V block is in and dP_j has been read.  With two stages
+            // (head_dim 128) dQ_j goes between them: the V block then arrives into
+            // the K half that dQ_j frees, while S_{j+1} and the elementwise warps'
+            // P phase proceed; with four stages dP_{j+1} goes first.
+            constexpr bool dq_mid = NS == 2;
             if (more) {
-              if (!mbar_wait_sleep(st_full((g + 1) % NS), ((g + 1) / NS) & 1, abort_flag)) { ok = false; break; }
-              if (!mbar_wait_sleep(rd, g & 1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(hf_full(s1, h1), par1, abort_flag)) { ok = false; break; }
+              if (!mbar_wait_sleep(rd_s, g & 1, abort_flag)) { ok = false; break; }
               tc_fence_after();
-              issue_sdp(T_S, lo_ra, (g + 1) % NS, 0);
+              issue_sdp(T_S, lo_ra, s1, h1);
               tc_commit(s_full);
-              issue_sdp(T_DP, lo_rb, (g + 1) % NS, 1);
-              tc_commit(dp_full);
-              if (j + 2 == it.nit) tc_commit(res_empty);
             }
+            auto issue_dp_next = [&]() -> bool {
+              if (!mbar_wait_sleep(hf_full(s1, h1 ^ 1), par1, abort_flag)) return false;
+              if (!mbar_wait_sleep(rd_dp, g & 1, abort_flag)) return false;
+              tc_fence_after();
+              issue_sdp(T_DP, lo_rb, s1, h1 ^ 1);
+              tc_commit(dp_full);
+              tc_commit(hf_empty(s1, h1 ^ 1));  // its V half
+              if (j + 2 == it.nit) tc_commit(res_empty);
+              return true;
+            };
+            if (more && !dq_mid && !issue_dp_next()) { ok = false; break; }
             // dQ += dS K   (dS in bf16 pairs from column T_DS, AB_COLS / 2 columns per warp)
             if (!mbar_wait_sleep(ds_full, g & 1, abort_flag)) { ok = false; break; }
             if (j == 0 && n > 0 && !mbar_wait_sleep(acc_empty, (n - 1) & 1, abort_flag)) { ok = false; break; }
             tc_fence_after();
-            issue_acc(T_A1, T_DS, AB_COLS / 2, lo_h0, j > 0);
+            issue_acc(T_A1, T_DS, AB_COLS / 2, lo_first, j > 0);
             tc_commit(ds_empty);
-            tc_commit(st_empty(s));
+            tc_commit(hf_empty(s, ha));  // the K half
+            if (more && dq_mid && !issue_dp_next()) { ok = false; break; }
           }
         }
         if (!ok) break;
@@ -442,9 +487,13 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
         float sv[C];
 #pragma unroll
         for (int c = 0; c < C; c += 32) TMEM_LD32(lane_addr + T_S + C * part + c, (reinterpret_cast<uint32_t*>(sv) + c));
+        tmem_wait_ld();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(rd_s);  // S of this block is in registers
         if (it.kv) {
-          tmem_wait_ld();
-          if (!mbar_wait_sleep(st_full(s), (g / NS) & 1, abort_flag)) { ok = false; break; }
+          // lse and D arrive with the block's Q half
+          if (!mbar_wait_sleep(hf_full(s, ha_of(g)), (g / NS) & 1, abort_flag)) { ok = false; break; }
           const float* vl = vec_base + s * 256 + C * part;   // lse / D of this warp's C queries
           // P^T = 2^(S^T * scale - lse[q])
 #pragma unroll
@@ -499,20 +548,28 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
           tc_fence_before();
           __syncwarp();
           if (lane == 0) {
-            mbar_arrive(rd);
+            mbar_arrive(rd_dp);
             mbar_arrive(ds_full);
           }
           ++gk;
         } else {
-          if (!mbar_wait_sleep(dp_full, g & 1, abort_flag)) { ok = false; break; }
-          tc_fence_after();
+          // With two stages dP_j is issued after dQ_{j-1} and may still be running:
+          // P first.  With four, dP_j has been issued beside S_j: read it first, so
+          // that dP_{j+1} can follow as early as before.
+          constexpr bool p_first = NS == 2;
           float dv[C];
+          auto load_dp = [&]() -> bool {
+            if (!mbar_wait_sleep(dp_full, g & 1, abort_flag)) return false;
+            tc_fence_after();
 #pragma unroll
-          for (int c = 0; c < C; c += 32) TMEM_LD32(lane_addr + T_DP + C * part + c, (reinterpret_cast<uint32_t*>(dv) + c));
-          tmem_wait_ld();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(rd);  // S and dP of this block are in registers
+            for (int c = 0; c < C; c += 32) TMEM_LD32(lane_addr + T_DP + C * part + c, (reinterpret_cast<uint32_t*>(dv) + c));
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rd_dp);  // dP of this block is in registers
+            return true;
+          };
+          if (!p_first && !load_dp()) { ok = false; break; }
           const float nl = -lse_r;
 #pragma unroll
           for (int i = 0; i < C; ++i) sv[i] = ex2_approx(fmaf(sv[i], sl2, nl));
@@ -524,6 +581,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
               if (c >= p.T || row >= p.T || c > row) sv[i] = 0.f;
             }
           }
+          if (p_first && !load_dp()) { ok = false; break; }
 #pragma unroll
           for (int i = 0; i < C; ++i) dv[i] = sv[i] * (dv[i] - d_r);
           uint32_t dw[C / 2];
