@@ -88,7 +88,7 @@ struct BwdSmem {
   static constexpr int STAGES = HD == 64 ? 4 : 2;
   static constexpr int RES_A = 0;                      // K (KV item) or Q (Q item)
   static constexpr int RES_B = KCH * CH;               // V or dO
-  static constexpr int HALF = KCH * CH;                // half of a stage: Q | dO (KV) or K | V (Q)
+  static constexpr int HALF = KCH * CH;                // half of a stage: one [128 rows][HD] tile
   static constexpr int ST_OFF = 2 * KCH * CH;
   static constexpr int STAGE = 2 * HALF;
   static constexpr int STG_OFF = ST_OFF + STAGES * STAGE;  // epilogue staging: one accumulator in bf16
@@ -317,7 +317,8 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       const uint32_t hi = desc_hi(1024);
       const uint32_t lo_ra = desc_lo(base + L::RES_A, 16), lo_rb = desc_lo(base + L::RES_B, 16);
       int g = 0, gk = 0, n = 0;
-      // S (from resident A and stage half 0) or dP (resident B, stage half 1) of the block in stage s
+      // S (resident A times the block's first operand) or dP (resident B times its second),
+      // the streamed operand in half `half` of stage s
       auto issue_sdp = [&](uint32_t dst, uint32_t lo_res, int s, int half) {
         const uint32_t lo_st = desc_lo(base + L::ST_OFF + s * L::STAGE + half * L::HALF, 16);
 #pragma unroll
@@ -328,7 +329,7 @@ __global__ void __launch_bounds__(AB_THREADS, 1) attn_bwd_kernel(const __grid_co
       };
       // accumulate A (bf16 pairs in TMEM from column a_col, each elementwise warp's
       // AB_COLS values of k packed at a_step * (k / AB_COLS) + (k % AB_COLS) / 2)
-      // times the stage half as MN-major B
+      // times a streamed operand as MN-major B
       constexpr int KPW = AB_COLS / 16;  // K16 steps per elementwise warp's columns
       auto issue_acc = [&](uint32_t dst, uint32_t a_col, uint32_t a_step, uint32_t lo_b, bool acc) {
 #pragma unroll
