@@ -104,6 +104,37 @@ def test_attention_forward_backward_match_oracle(B, T, H, hd):
         assert rel_fro(got, ref) < 1e-2, rel_fro(got, ref)
 
 
+@pytest.mark.parametrize("hd", [64, 128])
+def test_attention_backward_persistent_items_against_oracle(hd):
+    """More work items than SMs (each CTA of the persistent backward runs
+    several key-block and query-block items back to back), a last band of
+    heads narrower than the others and a ragged sequence length: dQ, dK and dV
+    against the oracle's causal attention backward."""
+    import torch
+    from paper_2510_14614_gb300 import fal
+    B, T, H = 3, 700, 6  # 6 blocks of 128 rows per sequence, 18 heads: 216 items
+    rng = np.random.default_rng(700 + hd)
+    d = H * hd
+    qkv = bf16_round(rng.standard_normal((B * T, 3 * d)))
+    dctx = bf16_round(rng.standard_normal((B * T, d)))
+    qkv_t = torch.as_tensor(qkv, dtype=torch.float32).to(torch.bfloat16).cuda()
+    dctx_t = torch.as_tensor(dctx, dtype=torch.float32).to(torch.bfloat16).cuda()
+    ctx_t, lse_t = fal.attention_fwd(qkv_t, B, T, H, hd)
+    dqkv_t = fal.attention_bwd(qkv_t, ctx_t, lse_t, dctx_t, B, T, H, hd)
+    dqkv_t2 = fal.attention_bwd(qkv_t, ctx_t, lse_t, dctx_t, B, T, H, hd)
+    torch.cuda.synchronize()
+    sp = lambda x: x.reshape(B, T, H, hd).transpose(0, 2, 1, 3)
+    mg = lambda x: x.transpose(0, 2, 1, 3).reshape(B * T, d)
+    q, k, v = (sp(t) for t in np.split(qkv, 3, axis=1))
+    ctx, p = O.causal_attention(q, k, v)
+    dq, dk, dv = O.causal_attention_backward(sp(dctx), q, k, v, p)
+    dqkv = dqkv_t.float().cpu().numpy()
+    for got, ref in ((dqkv[:, :d], mg(dq)), (dqkv[:, d:2 * d], mg(dk)), (dqkv[:, 2 * d:], mg(dv))):
+        assert rel_fro(got, ref) < 1e-2, rel_fro(got, ref)
+    # each item's sums run in a fixed order whichever CTA takes it: repeat calls agree bit for bit
+    np.testing.assert_array_equal(dqkv, dqkv_t2.float().cpu().numpy())
+
+
 def test_attention_backward_more_token_rows_than_a_grid_dimension():
     """B*T = 66560 token rows (above the 65535 limit of a grid's y and z
     dimensions) in short sequences: the kernel-level backward, including its
